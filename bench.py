@@ -1,0 +1,405 @@
+#!/usr/bin/env python
+"""Benchmark of the ECOKV prefill eviction pass (score -> select -> compact).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ecokv|reference] [--workload c3_b10]
+
+A step is one call of ecokv_evict over every layer and KV head of the
+workload (default: the 32768-token, 28-layer, 28/4-head Qwen2.5-VL-shaped
+video prefill, bf16, W = 8, pooling 5, budget 10 % = 3277 tokens/head), with
+K, V and the window queries already resident in HBM.  The inputs (1.88 GB of
+K and V) are larger than the 129 MB L2, so no flush is needed between steps.
+
+Metric: KV tokens processed per second per layer = L * H_kv * N / step time
+(every cached key row of every layer is scored; H_kv * (N - B) of them are
+evicted per layer).  One JSON line is printed by rank 0.
+
+--impl reference times the fp64 CPU oracle (the only other implementation of
+the method; the paper ships no code) on a bounded sample of the same workload.
+Under torchrun with N > 1 every rank runs its own replica (the (layer, head)
+units are independent: weak scaling, no data-path collective); the timing
+uses a barrier and the maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "KV tokens evicted/sec per layer at 1 GB300; % of HBM roofline (GB/s)"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ecokv", "reference"], default="ecokv")
+    ap.add_argument("--workload", default="c3_b10")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- byte model
+def byte_model(w) -> dict:
+    """Algorithmic bytes of one pass over the workload.
+
+    ALG (the roofline numerator): every K row read once, the window queries
+    read, the retained V rows read, the retained K and V rows written.
+    BL: the same plus a full read of V (the BASELINE formula).
+    """
+    e = w.elem_bytes
+    U = w.units
+    keep = min(w.budget, w.n)
+    k_bytes = U * w.n * w.d * e
+    q_bytes = w.n_layers * w.h_q * w.window * w.d * e
+    kept = U * keep * w.d * e
+    idx_bytes = U * keep * 4
+    alg = k_bytes + q_bytes + kept + 2 * kept + idx_bytes
+    bl = k_bytes + k_bytes + q_bytes + 2 * kept
+    return {"alg": alg, "bl": bl, "k": k_bytes, "q": q_bytes, "kept_rows": kept}
+
+
+def measured_peaks() -> tuple[float, str]:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_06663_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_record(workload: str):
+    """DRAM bytes per launch of the dominant kernel from a committed ncu
+    summary, valid only while the kernel sources are unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    r = rec.get(workload)
+    if not r or r.get("source_hash") != kernel_source_hash():
+        return None
+    return r
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        import tempfile
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.dev)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[4:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [r[0] for r in rows]
+        top = max(sm)
+        loaded = [r for r in rows if r[0] >= 0.5 * top] or rows
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in loaded:
+            for n, v in zip(names[1:], r[2][1:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": rows[0][1],
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- CPU oracle leg
+_INPUT_CACHE: dict = {}
+
+
+def _oracle_units(args):
+    """Worker: run the fp64 oracle on some (layer, head) units of a workload."""
+    wl_key, units = args
+    import torch
+    torch.set_num_threads(1)
+    from oracle import ecokv_oracle as O
+    from paper_2609_06663_gb300.workloads import make_inputs, workload
+    w = workload(wl_key)
+    n_tok = 0
+    t_total = 0.0
+    for (l, h) in units:
+        key = (wl_key, l)
+        if key not in _INPUT_CACHE:
+            _INPUT_CACHE.clear()
+            _INPUT_CACHE[key] = make_inputs(w, layers=range(l, l + 1))
+        K, V, Q = _INPUT_CACHE[key]
+        g = w.group
+        Ku, Vu, Qu = K[:, h:h + 1], V[:, h:h + 1], Q[:, h * g:(h + 1) * g]
+        p = O.Params(n_layers=1, h_kv=1, h_q=g, n=w.n, d=w.d, window=w.window, budget=w.budget,
+                     pool_kernel=w.pool_kernel)
+        t0 = time.perf_counter()
+        O.evict(Ku, Vu, Qu, p)
+        t_total += time.perf_counter() - t0
+        n_tok += w.n
+    return n_tok, t_total
+
+
+def oracle_pool(cores: int):
+    """A pool of spawned, single-threaded worker processes for the oracle."""
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[v] = "1"
+    return mp.get_context("spawn").Pool(cores)
+
+
+def cpu_oracle_rate(wl_key: str, w, n_units: int, pool, cores: int) -> dict:
+    """Tokens/s of the oracle over a bounded sample of units, split across
+    `cores` single-threaded workers that run in parallel."""
+    units = [((i // w.h_kv) % w.n_layers, i % w.h_kv) for i in range(n_units)]
+    per = [units[i::cores] for i in range(cores)]
+    per = [u for u in per if u]
+    t0 = time.perf_counter()
+    res = pool.map(_oracle_units, [(wl_key, u) for u in per])
+    wall = time.perf_counter() - t0
+    n_tok = sum(r[0] for r in res)
+    busy = max(r[1] for r in res)
+    return {"value": n_tok / busy, "unit": UNIT, "cores": len(per), "kind": "oracle",
+            "sample": f"{n_units} (layer, head) units of {w.name} ({n_tok} key rows), fp64 numpy oracle, "
+                      f"{len(per)} spawned single-thread workers; rate = rows / busiest worker's compute time "
+                      f"(input generation excluded); wall {wall:.1f} s"}
+
+
+def default_sample_units(w, cores: int) -> int:
+    # about 0.25 s of oracle time per 32k-token unit: aim for ~10-20 s of CPU work
+    per_unit = 0.25 * w.n / 32768 * max(1, w.group * w.window) / 56
+    return max(cores, min(4 * cores, int(15.0 / max(per_unit, 1e-3))))
+
+
+# ---------------------------------------------------------------- main
+def main():
+    args = parse_args()
+    import torch
+
+    from paper_2609_06663_gb300.workloads import workload
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    w = workload(args.workload)
+    cores = max(1, min(16, os.cpu_count() or 1))
+
+    if args.impl == "reference":
+        run_reference(args, w, rank, world, cores)
+        return
+
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2609_06663_gb300 import ecokv as E
+    from paper_2609_06663_gb300.workloads import make_inputs
+
+    import dataclasses
+    wr = dataclasses.replace(w, seed=w.seed + rank)
+    K, V, Q = make_inputs(wr, device=dev)
+    p = E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
+                      budget=w.budget, pool_kernel=w.pool_kernel)
+    ws = E.alloc_workspace(p, dev)
+    n_keep = min(w.budget, w.n)
+    idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
+    Ko = torch.empty(w.n_layers, w.h_kv, n_keep, w.d, dtype=K.dtype, device=dev)
+    Vo = torch.empty_like(Ko)
+    lam = torch.empty(w.n_layers, w.h_kv, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    dt = E.dtype_code(K)
+
+    def step():
+        code = E.ecokv_evict(p, dt, K, V, Q, idx, Ko, Vo, None, lam, ws, ws.numel(), stream)
+        if code:
+            raise E.EcokvError(code, "ecokv_evict")
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    assert E.ecokv_device_status(ws, stream) == 0
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    barrier()
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    tokens_step = w.units * w.n
+    value = world * tokens_step / (ms_step * 1e-3)
+
+    # end to end through the public API: pinned host inputs -> device -> pass -> host outputs
+    e2e = None
+    if rank == 0 or world > 1:
+        hK = K.cpu().pin_memory()
+        hV = V.cpu().pin_memory()
+        hQ = Q.cpu().pin_memory()
+        oidx = torch.empty(idx.shape, dtype=idx.dtype).pin_memory()
+        oK = torch.empty(Ko.shape, dtype=Ko.dtype).pin_memory()
+        oV = torch.empty(Vo.shape, dtype=Vo.dtype).pin_memory()
+
+        def e2e_step():
+            K.copy_(hK, non_blocking=True)
+            V.copy_(hV, non_blocking=True)
+            Q.copy_(hQ, non_blocking=True)
+            step()
+            oidx.copy_(idx, non_blocking=True)
+            oK.copy_(Ko, non_blocking=True)
+            oV.copy_(Vo, non_blocking=True)
+
+        e2e_step()
+        barrier()
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        a1.record(stream)
+        barrier()
+        e_ms = a0.elapsed_time(a1) / args.e2e_steps
+        if world > 1:
+            t = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_ms = float(t.item())
+        e2e = {"value": world * tokens_step / (e_ms * 1e-3), "unit": UNIT,
+               "h2d_bytes_per_step": int(hK.numel() * hK.element_size() + hV.numel() * hV.element_size()
+                                         + hQ.numel() * hQ.element_size()),
+               "d2h_bytes_per_step": int(oidx.numel() * 4 + oK.numel() * oK.element_size()
+                                         + oV.numel() * oV.element_size()),
+               "ms_per_step": e_ms}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    bm = byte_model(w)
+    peak, peak_kind = measured_peaks()
+    achieved = bm["alg"] / (ms_step * 1e-3) / 1e9
+    tr = traffic_record(args.workload)
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": tr["dram_bytes_per_launch"] if tr else None,
+                "kernel": "ecokv_evict pass (all launches of one call)",
+                "peak_kind": f"{peak_kind} copy bandwidth (hbm_gbs)",
+                "alg_bytes_per_launch": bm["alg"], "bl_bytes_per_launch": bm["bl"],
+                "bl_frac": round(bm["bl"] / (ms_step * 1e-3) / 1e9 / peak, 4)}
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        nu = args.cpu_sample_units or default_sample_units(w, cores)
+        with oracle_pool(cores) as pool:
+            cpu = cpu_oracle_rate(args.workload, w, nu, pool, cores)
+
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": round(ms_step, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded anisotropic + clustered/temporally correlated keys; no dataset)",
+        "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
+                   "evicted_rows_per_s": round(world * w.units * max(0, w.n - w.budget) / (ms_step * 1e-3), 1),
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": 4 * args.steps, "clocks": clocks,
+    }
+    print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_reference(args, w, rank: int, world: int, cores: int) -> None:
+    """The oracle timed as it stands, on host cores; rank 0 only."""
+    if rank != 0:
+        return
+    nu = args.cpu_sample_units or max(cores, 2 * cores)
+    rates = []
+    with oracle_pool(cores) as pool:
+        for i in range(args.warmup + args.steps):
+            r = cpu_oracle_rate(args.workload, w, nu, pool, cores)
+            if i >= args.warmup:
+                rates.append(r)
+    value = statistics.median(r["value"] for r in rates)
+    cpu = dict(rates[0])
+    cpu["value"] = value
+    out = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": round(w.units * w.n / value * 1e3, 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "f64", "data": "synthetic", "impl": "reference",
+           "config": {**w.describe(), "workload": w.name}, "cpu_baseline": cpu,
+           "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,146 @@
+/*
+ * ecokv.h - C ABI of libecokv.so, the GB300 (sm_103a) ECOKV prefill
+ * KV-cache eviction pass: score -> select -> compact.
+ *
+ * The method (ECOKV, "Geometry-Aware KV Cache Eviction via Complementary
+ * Diversity Metrics"): for every layer l and KV head h, each cached key-value
+ * pair i gets a score
+ *
+ *     S(i) = lambda * Stilde_div(i) + (1 - lambda) * S_imp(i)          (Eq. 7)
+ *
+ * where S_imp is the observation-window attention importance (SnapKV voting,
+ * Appendix A), Stilde_div the rescaled composite Euclidean/cosine diversity
+ * (Eq. 1-3 and the rescale of Sec. 5.2) and lambda the head-adaptive
+ * redundancy weight (Eq. 4-6).  The top (budget - window) non-window pairs by
+ * S are kept together with the whole observation window (Sec. 3 problem
+ * statement), and the kept K/V rows are gathered into a compact cache.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ *  - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *    never allocates device memory.  Scratch space is a caller-provided
+ *    workspace of at least ecokv_workspace_size() bytes.
+ *  - Layouts are dense row-major with d contiguous:
+ *        K, V    [n_layers][h_kv][n][d]        (dtype)
+ *        Qwin    [n_layers][h_q][window][d]    (dtype); row j of the window
+ *                 is the query at position n - window + j
+ *        S       [n_layers][h_kv][n - window]  float32 scores of the
+ *                 non-window candidates
+ *        lambda  [n_layers][h_kv]              float32
+ *        idx     [n_layers][h_kv][n_keep]      int32, n_keep = min(budget, n):
+ *                 the chosen candidates in ascending position, then the
+ *                 window positions n - window .. n - 1
+ *        K_out, V_out [n_layers][h_kv][n_keep][d] (dtype)
+ *  - Query head q belongs to KV head q / (h_q / h_kv).
+ *  - Pointers must be 16-byte aligned.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream).  Argument errors are detected on the host and returned
+ *    before anything is launched.  Errors found on the device (an index out of
+ *    range handed to ecokv_compact, a bounded wait that gave up) are recorded
+ *    in the workspace's status word; read them with ecokv_device_status().
+ *  - Calls that share a workspace must be ordered on one stream.
+ *  - Inputs must be finite; scores of non-finite inputs are unspecified.
+ */
+#ifndef ECOKV_H
+#define ECOKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ECOKV_OK = 0,
+  ECOKV_ERR_INVALID_ARG = 1,  /* bad sizes, null or misaligned pointers      */
+  ECOKV_ERR_UNSUPPORTED = 2,  /* valid request this build does not handle     */
+  ECOKV_ERR_WORKSPACE = 3,    /* workspace missing or smaller than required   */
+  ECOKV_ERR_CUDA = 4,         /* a CUDA runtime call failed                   */
+  ECOKV_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up           */
+  ECOKV_ERR_DEVICE_INDEX = 6  /* device saw an index outside [0, n)           */
+} ecokv_status;
+
+typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
+
+/* variant flags (ecokv_params.flags) */
+#define ECOKV_FLAG_SC_MIXKV_SIGN   0x1u /* s_C = -khat.mu (MixKV, Appendix A) instead of (1 - khat.mu)/2 */
+#define ECOKV_FLAG_LAMBDA_OVERRIDE 0x2u /* use lambda_override for every head (0 = SnapKV importance only) */
+
+typedef struct {
+  int32_t n_layers;    /* L >= 1 layers in one call                              */
+  int32_t h_kv;        /* KV heads per layer, >= 1                                */
+  int32_t h_q;         /* query heads per layer, a multiple of h_kv               */
+  int32_t n;           /* cached tokens N (Sec. 3: T), 1 <= n <= 2^24             */
+  int32_t d;           /* head dimension; this build supports d = 128             */
+  int32_t window;      /* observation window W (Sec. 5.3), 1 <= W <= min(n, budget);
+                          (h_q / h_kv) * W <= 256                                  */
+  int32_t budget;      /* B retained tokens per head, window included; B >= n keeps all */
+  int32_t pool_kernel; /* odd average-pooling width (Appendix A.3: 5)              */
+  float alpha;         /* Eq. 3 weight of the Euclidean diversity, in [0, 1] (0.8) */
+  float beta;          /* Eq. 6 weight of the Euclidean redundancy, in [0, 1] (0.6) */
+  float tau;           /* Eq. 5 temperature; <= 0 selects sqrt(d)                  */
+  float eps;           /* Eq. 2 min-max stabiliser, > 0 (1e-6)                     */
+  uint32_t flags;      /* ECOKV_FLAG_* bits                                        */
+  float lambda_override; /* lambda for every head when ECOKV_FLAG_LAMBDA_OVERRIDE  */
+} ecokv_params;
+
+/* Fill *p with the paper's defaults (Appendix A.3): alpha 0.8, beta 0.6,
+ * tau sqrt(d), eps 1e-6, pool_kernel 5, window 4, flags 0.  Shape fields are
+ * zeroed and must be set by the caller. */
+void ecokv_params_default(ecokv_params* p);
+
+/* Validate a parameter block.  Returns ECOKV_OK, ECOKV_ERR_INVALID_ARG (an
+ * impossible request: W > n, B < W, even pool_kernel, h_q % h_kv != 0,
+ * alpha/beta outside [0, 1], eps <= 0 ...) or ECOKV_ERR_UNSUPPORTED (d != 128,
+ * (h_q/h_kv)*W > 256, n > 2^24). */
+ecokv_status ecokv_check_params(const ecokv_params* p);
+
+/* Bytes of device workspace the calls below need for *p (0 if *p is invalid).
+ * The workspace holds per-chunk partial sums, per-head statistics, per-token
+ * importance / distance / cosine arrays and the status word. */
+size_t ecokv_workspace_size(const ecokv_params* p);
+
+/* Scores of every non-window candidate (Eq. 1-7) and the per-head lambda.
+ *   K, Qwin : inputs (dtype), see layouts above.
+ *   S       : out, float32 [L][h_kv][n - W].
+ *   lambda  : out, float32 [L][h_kv]; may be NULL.
+ *   dbg     : out, optional (may be NULL), float32 [L][h_kv][5][n - W] holding,
+ *             per candidate: raw window-attention sum, pooled importance S_imp,
+ *             Euclidean distance d_E, cosine khat.mu and composite S_div. */
+ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* Qwin,
+                         float* S, float* lambda, float* dbg, void* ws, size_t ws_bytes, void* stream);
+
+/* Per-head top-(B - W) selection over S (Sec. 3; ties go to the lower
+ * position) followed by the window: idx [L][h_kv][min(B, n)] int32.  Exact
+ * for any float32 S (radix select on the order-preserving integer image).
+ * ws may be NULL (no device status). */
+ecokv_status ecokv_select(const ecokv_params* p, const float* S, int32_t* idx, void* ws, size_t ws_bytes,
+                          void* stream);
+
+/* Gather the retained rows: K_out[l][h][r] = K[l][h][idx[l][h][r]], same for V.
+ * Bit-exact copies.  An idx entry outside [0, n) yields a zero row and, when
+ * ws is given, ECOKV_ERR_DEVICE_INDEX in the status word.  ws may be NULL. */
+ecokv_status ecokv_compact(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                           const int32_t* idx, void* K_out, void* V_out, void* ws, size_t ws_bytes,
+                           void* stream);
+
+/* The whole pass: score, select and compact in one call.  S and lambda are
+ * optional outputs (NULL to skip).  idx, K_out, V_out as above. */
+ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                         const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
+                         float* lambda, void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronise `stream`, then read and clear the workspace's device status
+ * word.  Returns ECOKV_OK, ECOKV_ERR_DEVICE_INDEX, ECOKV_ERR_TIMEOUT, or
+ * ECOKV_ERR_CUDA if the synchronisation itself failed. */
+ecokv_status ecokv_device_status(void* ws, void* stream);
+
+/* Static text for a status code. */
+const char* ecokv_status_string(ecokv_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ECOKV_H */

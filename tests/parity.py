@@ -1,0 +1,63 @@
+"""Comparison helpers for CUDA-path vs oracle parity (used by the gpu tests
+and smoke checks).  Tolerances: per-token scores within 1e-3 relative for
+bf16 inputs and 1e-5 for fp32 inputs, measured as
+|S_gpu - S_ref| <= tol * max(|S_ref|, mean_i |S_ref|); retained sets equal
+except for candidates whose oracle score lies within that tolerance of the
+oracle's k-th largest score; compacted rows bit-exact."""
+import numpy as np
+import torch
+
+from oracle import ecokv_oracle as O
+
+TOL = {"f32": 1e-5, "bf16": 1e-3}
+
+
+def oracle_params(p, **over) -> O.Params:
+    kw = {k: getattr(p, k) for k in ("n_layers", "h_kv", "h_q", "n", "d", "window", "budget", "pool_kernel",
+                                      "alpha", "beta", "tau", "eps", "flags", "lambda_override")}
+    kw.update(over)
+    return O.Params(**kw)
+
+
+def score_error(S_gpu: np.ndarray, S_ref: np.ndarray) -> float:
+    if S_ref.size == 0:
+        return 0.0
+    scale = np.maximum(np.abs(S_ref), np.abs(S_ref).mean())
+    scale = np.where(scale > 0, scale, 1.0)
+    return float((np.abs(S_gpu - S_ref) / scale).max())
+
+
+def check_scores(S_gpu, ref, tol, what=""):
+    err = score_error(np.asarray(S_gpu, dtype=np.float64), ref["S"])
+    assert err <= tol, f"{what}: score error {err:.3e} > {tol:g}"
+    return err
+
+
+def check_selection(idx_gpu: np.ndarray, ref: dict, p: O.Params, tol: float, what=""):
+    """Retained sets equal except for threshold ties within tolerance."""
+    n, w = p.n, p.window
+    idx_gpu = np.asarray(idx_gpu, dtype=np.int64)
+    assert idx_gpu.shape == (min(p.budget, n),), what
+    if p.budget >= n:
+        assert (idx_gpu == np.arange(n)).all(), what
+        return 0
+    k = p.budget - w
+    assert (idx_gpu[k:] == np.arange(n - w, n)).all(), f"{what}: window not retained at the end"
+    cand = idx_gpu[:k]
+    assert (np.diff(cand) > 0).all() if k > 1 else True, f"{what}: candidates not ascending"
+    assert ((cand >= 0) & (cand < n - w)).all(), what
+    if k == 0:
+        return 0
+    S = ref["S"]
+    thr = np.sort(S)[::-1][k - 1]
+    band = tol * max(abs(thr), np.abs(S).mean())
+    diff = set(cand.tolist()) ^ set(ref["idx"][:k].tolist())
+    bad = [i for i in diff if abs(S[i] - thr) > band]
+    assert not bad, f"{what}: {len(bad)} retained-set differences outside the threshold band, e.g. {bad[:5]}"
+    return len(diff)
+
+
+def check_rows(K: torch.Tensor, idx: torch.Tensor, K_out: torch.Tensor, what=""):
+    """K_out[r] must be a bit-exact copy of K[idx[r]]."""
+    ref = K[idx.long().cpu()] if K.device.type == "cpu" else K[idx.long()]
+    assert torch.equal(K_out.to(ref.device), ref), f"{what}: compacted rows differ"

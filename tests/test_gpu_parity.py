@@ -1,0 +1,182 @@
+"""CUDA path (through the C ABI) vs the fp64 oracle on the same seeded inputs.
+
+Small shapes span several 128-key chunks and a ragged tail; the configs run
+at their own shapes (layer subsets where the oracle would take long), and the
+32k-token config runs at full size in the same launch the benchmark times,
+checked on sampled (layer, head) units."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import ecokv_oracle as O
+from paper_2609_06663_gb300 import ecokv as E
+from paper_2609_06663_gb300.workloads import CONFIGS, make_inputs, small_workload, sweep_workload, workload
+from tests.parity import TOL, check_rows, check_scores, check_selection, oracle_params, score_error
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def params_of(w, **kw):
+    return E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
+                         budget=w.budget, pool_kernel=w.pool_kernel, **kw)
+
+
+def run_and_compare(w, layers=None, units=None, **kw):
+    """Score + evict + split select on the GPU; compare with the oracle."""
+    K, V, Q = make_inputs(w, layers=layers)
+    nl = K.shape[0]
+    wl = type(w)(**{**{f: getattr(w, f) for f in w.__dataclass_fields__}, "n_layers": nl})
+    p = params_of(wl, **kw)
+    Kd, Vd, Qd = K.to(DEV), V.to(DEV), Q.to(DEV)
+    ws = E.alloc_workspace(p, DEV)
+    S, lam, dbg = E.score(p, Kd, Qd, ws=ws, dbg=True)
+    idx, Ko, Vo, S2, lam2 = E.evict(p, Kd, Vd, Qd, ws=ws, want_scores=True)
+    idx_sel = E.select(p, S)
+    torch.cuda.synchronize()
+    assert E.ecokv_device_status(ws) == 0
+    # fused entry == split entries, bit for bit
+    assert torch.equal(S, S2) and torch.equal(lam, lam2) and torch.equal(idx, idx_sel)
+    op = oracle_params(p)
+    units = units or [(l, h) for l in range(nl) for h in range(w.h_kv)]
+    ref = O.evict(K, V, Q, op, heads=units)
+    tol = TOL[w.dtype]
+    S_np, D_np = S.cpu().double().numpy(), dbg.cpu().double().numpy()
+    worst = 0.0
+    for (l, h) in units:
+        r = ref[(l, h)]
+        what = f"{w.name} unit ({l},{h})"
+        worst = max(worst, check_scores(S_np[l, h], r, tol, what))
+        assert abs(float(lam[l, h]) - r["lam"]) <= tol, what
+        if p.n > p.window:
+            assert score_error(D_np[l, h, 1], r["s_imp"]) <= tol, what + " S_imp"
+            assert score_error(D_np[l, h, 2], r["d_e"]) <= tol, what + " d_E"
+            assert np.abs(D_np[l, h, 3] - r["c"]).max() <= tol, what + " cosine"
+            assert score_error(D_np[l, h, 4], r["s_div"]) <= tol, what + " S_div"
+        # select is exact given the same fp32 scores
+        exact = O.select(S_np[l, h], op)
+        assert (idx_sel[l, h].cpu().numpy() == exact).all(), what + " select"
+        check_selection(idx[l, h].cpu().numpy(), r, op, tol, what)
+        check_rows(Kd[l, h], idx[l, h], Ko[l, h], what)
+        check_rows(Vd[l, h], idx[l, h], Vo[l, h], what)
+    return worst
+
+
+SMALL = [
+    dict(n=1000, h_kv=2, group=1, window=8, budget=100, pool_kernel=7, dtype="f32"),
+    dict(n=1000, h_kv=2, group=4, window=4, budget=100, pool_kernel=5, dtype="bf16", clustered=True),
+    dict(n=129, h_kv=1, group=2, window=1, budget=17, pool_kernel=1, dtype="f32"),
+    dict(n=127, h_kv=3, group=1, window=3, budget=30, pool_kernel=3, dtype="bf16"),
+    dict(n=600, h_kv=1, group=8, window=32, budget=120, pool_kernel=5, dtype="bf16"),   # g*W = 256
+    dict(n=600, h_kv=1, group=8, window=32, budget=120, pool_kernel=5, dtype="f32"),
+    dict(n=300, h_kv=2, group=2, window=5, budget=5, pool_kernel=5, dtype="f32"),       # B == W
+    dict(n=200, h_kv=2, group=1, window=4, budget=250, pool_kernel=5, dtype="bf16"),    # B >= N
+    dict(n=8, h_kv=2, group=1, window=8, budget=8, pool_kernel=5, dtype="f32"),         # N == W
+    dict(n=1, h_kv=1, group=1, window=1, budget=1, pool_kernel=1, dtype="f32"),         # N == 1
+    dict(n=2, h_kv=1, group=3, window=1, budget=1, pool_kernel=3, dtype="bf16"),
+    dict(n=5000, h_kv=2, group=7, window=8, budget=500, pool_kernel=5, dtype="bf16", n_layers=2,
+         clustered=True),
+]
+
+
+@pytest.mark.parametrize("case", SMALL, ids=lambda c: f"n{c['n']}_g{c['group']}_w{c['window']}_b{c['budget']}_{c['dtype']}")
+def test_small_shapes(case):
+    run_and_compare(small_workload(seed=11, **case))
+
+
+@pytest.mark.parametrize("flags,extra", [
+    (O.FLAG_SC_MIXKV_SIGN, dict(alpha=0.0, beta=0.0)),          # MixKV special case
+    (O.FLAG_LAMBDA_OVERRIDE, dict(lambda_override=0.0)),         # SnapKV importance only
+    (0, dict(alpha=1.0, beta=1.0, tau=3.0)),
+])
+def test_variants(flags, extra):
+    w = small_workload(n=777, h_kv=2, group=2, window=4, budget=64, dtype="f32", seed=5, clustered=True)
+    run_and_compare(w, flags=flags, **extra)
+
+
+def test_config_c0_full():
+    run_and_compare(CONFIGS["c0"])
+
+
+@pytest.mark.parametrize("key", ["c1_b10", "c1_b20"])
+def test_config_c1_two_layers(key):
+    run_and_compare(CONFIGS[key], layers=range(0, 2))
+
+
+def test_config_c2_two_layers():
+    run_and_compare(CONFIGS["c2"], layers=range(5, 7))
+
+
+@pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4)])
+def test_sweep_points(n, window):
+    run_and_compare(sweep_workload(n, window))
+
+
+def test_identical_keys_all_ties():
+    # every key equal: d_E and the cosine are constant, S ties wherever the
+    # pooled importance ties; the selection must still be exact.
+    w = small_workload(n=400, h_kv=1, group=2, window=4, budget=40, dtype="bf16")
+    K, V, Q = make_inputs(w)
+    K[:] = K[:, :, :1]
+    p = params_of(w)
+    Kd, Vd, Qd = K.to(DEV), V.to(DEV), Q.to(DEV)
+    idx, Ko, Vo, S, lam = E.evict(p, Kd, Vd, Qd, want_scores=True)
+    ref = O.evict(K, V, Q, oracle_params(p))[(0, 0)]
+    check_scores(S[0, 0].cpu().double().numpy(), ref, TOL["bf16"], "identical keys")
+    assert (idx[0, 0].cpu().numpy() == O.select(S[0, 0].cpu().double().numpy(), oracle_params(p))).all()
+
+
+@pytest.mark.parametrize("n,window,budget", [(5000, 4, 300), (300, 1, 299), (70000, 8, 7000)])
+def test_select_exact_on_crafted_scores(n, window, budget):
+    # ties, negatives, +-0: radix select must equal (S desc, position asc)
+    g = torch.Generator().manual_seed(n)
+    tv = n - window
+    S = (torch.randint(-6, 7, (2, 3, tv), generator=g).float() / 4)
+    S[0, 0, ::7] = -0.0
+    S[1, 2] = 1.5                                     # one head all ties
+    p = E.make_params(n_layers=2, h_kv=3, h_q=3, n=n, window=window, budget=budget)
+    idx = E.select(p, S.to(DEV)).cpu().numpy()
+    op = oracle_params(p)
+    for l in range(2):
+        for h in range(3):
+            assert (idx[l, h] == O.select(S[l, h].double().numpy(), op)).all()
+
+
+def test_compact_reports_bad_index():
+    w = small_workload(n=300, h_kv=2, group=1, window=4, budget=40, dtype="bf16")
+    K, V, Q = make_inputs(w)
+    p = params_of(w)
+    Kd, Vd = K.to(DEV), V.to(DEV)
+    idx = torch.arange(40, dtype=torch.int32, device=DEV).repeat(1, 2, 1).contiguous()
+    idx[0, 1, 7] = 300                                   # out of range: zero row + status
+    ws = E.alloc_workspace(p, DEV)
+    Ko, Vo = E.compact(p, Kd, Vd, idx, ws=ws)
+    assert E.ecokv_device_status(ws) == 6
+    assert E.ecokv_device_status(ws) == 0              # cleared by the read
+    assert torch.count_nonzero(Ko[0, 1, 7]) == 0 and torch.count_nonzero(Vo[0, 1, 7]) == 0
+    good = idx[0, 0].long()
+    assert torch.equal(Ko[0, 0], Kd[0, 0][good])
+
+
+def test_c3_full_size_sampled_units():
+    # the 32k-token, 28-layer workload exactly as the benchmark launches it
+    w = workload("c3_b10")
+    K, V, Q = make_inputs(w, device=DEV)
+    p = params_of(w)
+    ws = E.alloc_workspace(p, DEV)
+    idx, Ko, Vo, S, lam = E.evict(p, K, V, Q, ws=ws, want_scores=True)
+    torch.cuda.synchronize()
+    assert E.ecokv_device_status(ws) == 0
+    units = [(0, 0), (13, 2), (27, 3)]
+    op = oracle_params(p, n_layers=1)
+    for (l, h) in units:
+        Kh = K[l:l + 1, h:h + 1].cpu()
+        Qh = Q[l:l + 1, h * w.group:(h + 1) * w.group].cpu()
+        r = O.evict(Kh, Kh, Qh, oracle_params(p, n_layers=1, h_kv=1, h_q=w.group))[(0, 0)]
+        what = f"c3 unit ({l},{h})"
+        check_scores(S[l, h].cpu().double().numpy(), r, TOL["bf16"], what)
+        check_selection(idx[l, h].cpu().numpy(), r, oracle_params(p, n_layers=1, h_kv=1, h_q=w.group),
+                        TOL["bf16"], what)
+        check_rows(K[l, h], idx[l, h], Ko[l, h], what)
+        check_rows(V[l, h], idx[l, h], Vo[l, h], what)
+    del op
