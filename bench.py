@@ -72,6 +72,15 @@ def byte_model(w) -> dict:
     return {"alg": alg, "bl": bl, "k": k_bytes, "q": q_bytes, "kept_rows": kept}
 
 
+def launches_per_call(w) -> int:
+    """Kernels one ecokv_evict call launches: the persistent tensor-core
+    streaming kernel (bf16, n >= 128, g*W <= 124) or the two CUDA-core passes,
+    then the finalize/select/compact kernel."""
+    r = w.group * w.window
+    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 4 <= 128
+    return 2 if tc else 3
+
+
 def measured_peaks() -> tuple[float, str]:
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -371,7 +380,7 @@ def main():
                    "evicted_rows_per_s": round(world * w.units * max(0, w.n - w.budget) / (ms_step * 1e-3), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-        "gpu_launches": 4 * args.steps, "clocks": clocks,
+        "gpu_launches": launches_per_call(w) * args.steps, "clocks": clocks,
     }
     print(json.dumps(out))
     if world > 1:

@@ -66,6 +66,7 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
 /* variant flags (ecokv_params.flags) */
 #define ECOKV_FLAG_SC_MIXKV_SIGN   0x1u /* s_C = -khat.mu (MixKV, Appendix A) instead of (1 - khat.mu)/2 */
 #define ECOKV_FLAG_LAMBDA_OVERRIDE 0x2u /* use lambda_override for every head (0 = SnapKV importance only) */
+#define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 
 typedef struct {
   int32_t n_layers;    /* L >= 1 layers in one call                              */

@@ -1,33 +1,43 @@
-// C ABI of libecokv.so: argument checks, workspace layout and launches.
-// Every entry point validates on the host and returns before launching
-// anything when an argument is wrong.
+// C ABI of libecokv.so: argument checks, workspace layout, path choice and
+// launches.  Every entry point validates on the host and returns before
+// launching anything when an argument is wrong.
+//
+// Paths.  bf16 inputs with n >= 128 and (h_q/h_kv)*W <= 124 stream K through
+// the persistent tensor-core kernel (tc_pass.cu, one launch for both passes);
+// fp32 inputs, other shapes and calls with ECOKV_FLAG_FORCE_SIMT use the
+// CUDA-core passes (score_simt.cu, two launches).  Either way one more launch
+// (finalize_select.cu) turns the pass-2 outputs into scores, selects and
+// gathers the kept rows.
 
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "ecokv_internal.cuh"
+#include "tc_pass.cuh"
 
 namespace ecokv {
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-Layout make_layout(const ecokv_params& p) {
+Layout make_layout(const ecokv_params& p, int chunk) {
   Layout L{};
   L.U = p.n_layers * p.h_kv;
   L.R = (p.h_q / p.h_kv) * p.window;
   L.N = p.n;
   L.W = p.window;
   L.Tv = p.n - p.window;
-  L.nchunks = (p.n + kChunk - 1) / kChunk;
+  L.chunk = chunk;
+  L.nchunks = (p.n + chunk - 1) / chunk;
   L.p1_stride = 2 * L.R + 2 * kD;
   L.ustat_stride = (2 * kD + 2 + L.R + 3) & ~3;
   const size_t U = (size_t)L.U;
   size_t off = 0;
   L.status = off;  off += 256;
-  L.cnt = off;     off += align256(U * 4);
+  L.sync = off;    L.sync_bytes = (4 + 4 * U) * 4;  off += align256(L.sync_bytes);
   L.p1part = off;  off += align256(U * L.nchunks * L.p1_stride * 4);
   L.ustat = off;   off += align256(U * L.ustat_stride * 4);
-  L.p2part = off;  off += align256(U * L.nchunks * 4);
+  L.p2part = off;  off += align256(U * L.nchunks * kP2Stride * 4);
   L.simp = off;    off += align256(U * L.Tv * 4);
   L.dE = off;      off += align256(U * L.Tv * 4);
   L.cosv = off;    off += align256(U * L.Tv * 4);
@@ -38,10 +48,28 @@ Layout make_layout(const ecokv_params& p) {
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+static size_t workspace_bytes(const ecokv_params& p) {
+  const size_t a = make_layout(p, kChunk).total, b = make_layout(p, kTcChunk).total;
+  return a > b ? a : b;
+}
+
 static ecokv_status check_ws(const ecokv_params* p, void* ws, size_t ws_bytes) {
   if (ws == nullptr || !aligned16(ws)) return ECOKV_ERR_WORKSPACE;
-  if (ws_bytes < make_layout(*p).total) return ECOKV_ERR_WORKSPACE;
+  if (ws_bytes < workspace_bytes(*p)) return ECOKV_ERR_WORKSPACE;
   return ECOKV_OK;
+}
+
+static bool use_tensor_path(const ecokv_params& p, ecokv_dtype dt) {
+  if (dt != ECOKV_BF16 || (p.flags & ECOKV_FLAG_FORCE_SIMT)) return false;
+  if (p.n < 128) return false;
+  return tc_rows_half((p.h_q / p.h_kv) * p.window) > 0;
+}
+
+static int env_int(const char* name, int dflt, int lo, int hi) {
+  const char* v = getenv(name);
+  if (v == nullptr || *v == 0) return dflt;
+  const int x = atoi(v);
+  return x < lo ? lo : (x > hi ? hi : x);
 }
 
 static ScoreArgs score_args(const ecokv_params& p, const Layout& L, const void* K, const void* Q, char* ws) {
@@ -61,7 +89,7 @@ static ScoreArgs score_args(const ecokv_params& p, const Layout& L, const void* 
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
   a.p1part = reinterpret_cast<float*>(ws + L.p1part);
   a.ustat = reinterpret_cast<float*>(ws + L.ustat);
-  a.cnt = reinterpret_cast<unsigned*>(ws + L.cnt);
+  a.cnt = reinterpret_cast<unsigned*>(ws + L.sync) + 4;
   a.p2part = reinterpret_cast<float*>(ws + L.p2part);
   a.simp = reinterpret_cast<float*>(ws + L.simp);
   a.dE = reinterpret_cast<float*>(ws + L.dE);
@@ -95,10 +123,63 @@ static FinalArgs final_args(const ecokv_params& p, const Layout& L, char* ws) {
   return f;
 }
 
-// Run both streaming passes: fills the per-token arrays and unit statistics.
-static ecokv_status run_passes(const ecokv_params& p, const Layout& L, ecokv_dtype dt, const void* K,
-                               const void* Q, char* ws, cudaStream_t s) {
-  if (cudaMemsetAsync(ws + L.cnt, 0, (size_t)L.U * 4, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+static CompactArgs compact_args(const ecokv_params& p, const void* K, const void* V, const int32_t* idx, void* Ko,
+                                void* Vo, unsigned* status) {
+  CompactArgs c{};
+  c.K = K;
+  c.V = V;
+  c.idx = idx;
+  c.K_out = Ko;
+  c.V_out = Vo;
+  c.N = p.n;
+  c.n_keep = p.budget < p.n ? p.budget : p.n;
+  c.status = status;
+  return c;
+}
+
+// Both streaming passes on the tensor cores in one launch (after clearing
+// the per-call counters).
+static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
+  const Layout L = make_layout(p, kTcChunk);
+  if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  TcArgs a{};
+  a.U = L.U;
+  a.N = p.n;
+  a.W = p.window;
+  a.R = L.R;
+  a.R4 = (L.R + 3) & ~3;
+  a.NP = 2 * tc_rows_half(L.R);
+  a.g = p.h_q / p.h_kv;
+  a.h_kv = p.h_kv;
+  a.h_q = p.h_q;
+  a.Tv = L.Tv;
+  a.tiles_per_chunk = kTcTilesPerChunk;
+  a.nchunks = L.nchunks;
+  a.lag_p2 = env_int("ECOKV_LAG_P2", 4, 1, 64);
+  a.step_items = 2 * a.nchunks;
+  a.total_tickets = (L.U + a.lag_p2) * a.step_items;
+  a.p1_stride = L.p1_stride;
+  a.ustat_stride = L.ustat_stride;
+  a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
+  a.timeout_cycles = 4000000000LL;  // about 2 s of SM clock per wait
+  a.Q = Q;
+  a.p1part = reinterpret_cast<float*>(ws + L.p1part);
+  a.ustat = reinterpret_cast<float*>(ws + L.ustat);
+  a.p2part = reinterpret_cast<float*>(ws + L.p2part);
+  a.simp = reinterpret_cast<float*>(ws + L.simp);
+  a.dE = reinterpret_cast<float*>(ws + L.dE);
+  a.cosv = reinterpret_cast<float*>(ws + L.cosv);
+  a.sync = reinterpret_cast<unsigned*>(ws + L.sync);
+  a.status = reinterpret_cast<unsigned*>(ws + L.status);
+  if (launch_tc(K, a, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  return ECOKV_OK;
+}
+
+// CUDA-core streaming passes: fill the per-token arrays and unit statistics.
+static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const void* K, const void* Q, char* ws,
+                                    cudaStream_t s) {
+  const Layout L = make_layout(p, kChunk);
+  if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   const ScoreArgs a = score_args(p, L, K, Q, ws);
   if (launch_score_simt(a, dt, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
@@ -131,18 +212,20 @@ ecokv_status ecokv_check_params(const ecokv_params* p) {
   if (p->pool_kernel < 1 || (p->pool_kernel & 1) == 0) return ECOKV_ERR_INVALID_ARG;
   if (!(p->alpha >= 0.f && p->alpha <= 1.f) || !(p->beta >= 0.f && p->beta <= 1.f)) return ECOKV_ERR_INVALID_ARG;
   if (!(p->eps > 0.f) || !isfinite(p->eps) || !isfinite(p->tau)) return ECOKV_ERR_INVALID_ARG;
-  if ((p->flags & ~(ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE)) != 0u) return ECOKV_ERR_INVALID_ARG;
+  const uint32_t known = ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_FORCE_SIMT;
+  if ((p->flags & ~known) != 0u) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_LAMBDA_OVERRIDE) && !isfinite(p->lambda_override)) return ECOKV_ERR_INVALID_ARG;
   if (p->d != kD) return ECOKV_ERR_UNSUPPORTED;
   if (p->n > kMaxN) return ECOKV_ERR_UNSUPPORTED;
   if ((long long)(p->h_q / p->h_kv) * p->window > kMaxRows) return ECOKV_ERR_UNSUPPORTED;
   if ((long long)p->n_layers * p->h_kv > (1 << 20)) return ECOKV_ERR_UNSUPPORTED;
+  if ((long long)p->n_layers * p->h_kv * p->n > (1LL << 31) / kD) return ECOKV_ERR_UNSUPPORTED;
   return ECOKV_OK;
 }
 
 size_t ecokv_workspace_size(const ecokv_params* p) {
   if (ecokv_check_params(p) != ECOKV_OK) return 0;
-  return make_layout(*p).total;
+  return workspace_bytes(*p);
 }
 
 ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* Qwin, float* S,
@@ -154,15 +237,17 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   if (p->n > p->window && (!S || !aligned16(S))) return ECOKV_ERR_INVALID_ARG;
   if ((lambda && ((uintptr_t)lambda & 3u)) || (dbg && !aligned16(dbg))) return ECOKV_ERR_INVALID_ARG;
   if ((st = check_ws(p, ws, ws_bytes)) != ECOKV_OK) return st;
-  const Layout L = make_layout(*p);
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = run_passes(*p, L, dtype, K, Qwin, w, s)) != ECOKV_OK) return st;
+  const bool tc = use_tensor_path(*p, dtype);
+  const Layout L = make_layout(*p, tc ? kTcChunk : kChunk);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.lambda = lambda;
   f.dbg = dbg;
-  if (launch_finalize(f, L.U, true, false, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
+  if (st != ECOKV_OK) return st;
+  if (launch_finalize(f, nullptr, dtype, L.U, false, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
 }
 
@@ -174,11 +259,11 @@ ecokv_status ecokv_select(const ecokv_params* p, const float* S, int32_t* idx, v
   if (st != ECOKV_OK) return st;
   if (!idx || !aligned16(idx)) return ECOKV_ERR_INVALID_ARG;
   if (p->budget < p->n && p->n > p->window && (!S || !aligned16(S))) return ECOKV_ERR_INVALID_ARG;
-  const Layout L = make_layout(*p);
+  const Layout L = make_layout(*p, kChunk);
   FinalArgs f = final_args(*p, L, nullptr);
   f.S = const_cast<float*>(S);
   f.idx = idx;
-  if (launch_finalize(f, L.U, false, true, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
+  if (launch_select(f, L.U, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
 }
 
@@ -191,16 +276,9 @@ ecokv_status ecokv_compact(const ecokv_params* p, ecokv_dtype dtype, const void*
   if (!aligned16(K) || !aligned16(V) || !aligned16(K_out) || !aligned16(V_out) || ((uintptr_t)idx & 3u))
     return ECOKV_ERR_INVALID_ARG;
   if (ws != nullptr && (!aligned16(ws) || ws_bytes < 256)) return ECOKV_ERR_WORKSPACE;
-  const Layout L = make_layout(*p);
-  CompactArgs c{};
-  c.K = K;
-  c.V = V;
-  c.idx = idx;
-  c.K_out = K_out;
-  c.V_out = V_out;
-  c.N = p->n;
-  c.n_keep = p->budget < p->n ? p->budget : p->n;
-  c.status = ws ? reinterpret_cast<unsigned*>(static_cast<char*>(ws) + L.status) : nullptr;
+  const Layout L = make_layout(*p, kChunk);
+  unsigned* status = ws ? reinterpret_cast<unsigned*>(static_cast<char*>(ws) + L.status) : nullptr;
+  const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, status);
   if (launch_compact(c, dtype, L.U, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
 }
@@ -217,25 +295,19 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
     return ECOKV_ERR_INVALID_ARG;
   if ((S && !aligned16(S)) || (lambda && ((uintptr_t)lambda & 3u))) return ECOKV_ERR_INVALID_ARG;
   if ((st = check_ws(p, ws, ws_bytes)) != ECOKV_OK) return st;
-  const Layout L = make_layout(*p);
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = run_passes(*p, L, dtype, K, Qwin, w, s)) != ECOKV_OK) return st;
+  const bool tc = use_tensor_path(*p, dtype);
+  const Layout L = make_layout(*p, tc ? kTcChunk : kChunk);
   FinalArgs f = final_args(*p, L, w);
-  f.S = S ? S : reinterpret_cast<float*>(w + L.sbuf);
+  f.S = S;
+  f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);
   f.lambda = lambda;
   f.idx = idx;
-  if (launch_finalize(f, L.U, true, true, s) != cudaSuccess) return ECOKV_ERR_CUDA;
-  CompactArgs c{};
-  c.K = K;
-  c.V = V;
-  c.idx = idx;
-  c.K_out = K_out;
-  c.V_out = V_out;
-  c.N = p->n;
-  c.n_keep = f.n_keep;
-  c.status = reinterpret_cast<unsigned*>(w + L.status);
-  if (launch_compact(c, dtype, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, reinterpret_cast<unsigned*>(w + L.status));
+  st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
+  if (st != ECOKV_OK) return st;
+  if (launch_finalize(f, &c, dtype, L.U, true, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
 }
 

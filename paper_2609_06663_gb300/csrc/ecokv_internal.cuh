@@ -14,6 +14,18 @@ constexpr int kD = 128;          // supported head dimension
 constexpr int kMaxRows = 256;    // max (h_q / h_kv) * window
 constexpr int kChunk = 128;      // keys per chunk of the streaming passes
 constexpr int kMaxN = 1 << 24;
+constexpr int kP2Stride = 8;     // floats per (unit, chunk) pass-2 partial, see P2_* below
+constexpr int kSmemScores = 48 * 1024;  // candidates whose scores the finaliser keeps in shared memory
+
+// pass-2 partial record of one (unit, chunk)
+enum : int {
+  P2_SUM_DE_ALL = 0,  // sum of d_E over the chunk's keys i < N (Eq. 4 uses all T keys)
+  P2_MIN_DE = 1,      // min of d_E over candidates i < N - W (+inf if none)
+  P2_MAX_DE = 2,      // max of d_E over candidates (-inf if none)
+  P2_SUM_DE = 3,      // sum of d_E over candidates
+  P2_SUM_COS = 4,     // sum of khat . mu over candidates
+  P2_SUM_RAW = 5      // sum of the raw importance vote over candidates
+};
 
 // Device status word (first bytes of the workspace).
 struct DevStatus {
@@ -21,18 +33,22 @@ struct DevStatus {
   unsigned detail;   // unit or item that raised it
 };
 
-// Byte offsets of the workspace regions for one parameter block.
+// Byte offsets of the workspace regions for one parameter block and one
+// streaming chunk size (kChunk keys on the CUDA-core path, kTcChunk on the
+// tensor-core path).
 struct Layout {
   int U;             // units = n_layers * h_kv
   int R;             // window rows per unit = (h_q / h_kv) * window
   int N, W, Tv;      // tokens, window, candidates
-  int nchunks;       // ceil(N / kChunk)
+  int chunk;         // keys per streaming chunk
+  int nchunks;       // ceil(N / chunk)
   int p1_stride;     // floats per (unit, chunk) pass-1 partial: 2R + 2D
   int ustat_stride;  // floats per unit statistics record
-  size_t status, cnt, p1part, ustat, p2part, simp, dE, cosv, sbuf, total;
+  size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, total;
+  size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
 
-Layout make_layout(const ecokv_params& p);
+Layout make_layout(const ecokv_params& p, int chunk);
 
 // unit statistics record (floats):  [0,D) kbar | [D,2D) mu | [2D] ||kbar||^2 |
 //                                    [2D+1] ||mu||^2 | [2D+2, 2D+2+R) log2-LSE of the window rows
@@ -49,7 +65,7 @@ struct ScoreArgs {
   float scale_log2;  // log2(e) / sqrt(d): logits are kept in log2 units
   float* p1part;
   float* ustat;
-  unsigned* cnt;
+  unsigned* cnt;     // per-unit pass-1 arrival counters
   float* p2part;
   float* simp;
   float* dE;
@@ -61,12 +77,13 @@ struct FinalArgs {
   float alpha, beta, tau, eps, lambda_override;
   unsigned flags;
   int n_keep;
-  const float* p2part;
+  const float* p2part;  // [U][nchunks][kP2Stride]
   const float* ustat;
   const float* simp;
   const float* dE;
   const float* cosv;
-  float* S;          // [U][Tv] scores (output of finalize, input of select)
+  float* S;          // [U][Tv] scores out, or null
+  float* S_scratch;  // [U][Tv] workspace scores, used when S is null and Tv > kSmemScores
   float* lambda;     // [U] or null
   float* dbg;        // [U][5][Tv] or null
   int32_t* idx;      // [U][n_keep] or null
@@ -84,7 +101,11 @@ struct CompactArgs {
 
 // launchers (return cudaGetLastError() after the launch)
 cudaError_t launch_score_simt(const ScoreArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
-cudaError_t launch_finalize(const FinalArgs& a, int U, bool do_score, bool do_select, cudaStream_t s);
+// finalize (scores), then optionally select and gather, one CTA per unit
+cudaError_t launch_finalize(const FinalArgs& f, const CompactArgs* c, ecokv_dtype dt, int U, bool do_select,
+                            cudaStream_t s);
+// select only, on caller scores f.S
+cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s);
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
 
 }  // namespace ecokv

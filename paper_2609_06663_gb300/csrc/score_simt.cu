@@ -171,6 +171,38 @@ __device__ void rows_max_expsum(float (&x)[RB], float* red, float* mrow, float* 
   __syncthreads();
 }
 
+__device__ __forceinline__ float warp_min(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float block_min128(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_min(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float s = red[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) s = fminf(s, red[w]);
+  __syncthreads();
+  return s;
+}
+
+__device__ __forceinline__ float block_max128(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_max(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float s = red[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) s = fmaxf(s, red[w]);
+  __syncthreads();
+  return s;
+}
+
 __device__ __forceinline__ float block_sum128(float v, float* red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   v = warp_sum(v);
@@ -276,7 +308,6 @@ __global__ void __launch_bounds__(kThreads) pass1_kernel(ScoreArgs a) {
   if (t == 0) {
     us[ustat_ksq()] = ksq;
     us[ustat_musq()] = msq;
-    a.cnt[u] = 0u;
   }
 }
 
@@ -316,14 +347,28 @@ __global__ void __launch_bounds__(kThreads) pass2_kernel(ScoreArgs a) {
   dist_and_dot<T>(krow, kbar, mu, &d2, &dmu);
   const float dE = sqrtf(d2);
   const float cosv = dmu * (1.f / fmaxf(sqrtf(nrm2), 1e-12f));
-  if (i < a.Tv) {
+  const bool cand = i < a.Tv;
+  if (cand) {
     const size_t o = (size_t)u * a.Tv + i;
     a.simp[o] = vote;
     a.dE[o] = dE;
     a.cosv[o] = cosv;
   }
-  const float s = block_sum128(valid ? dE : 0.f, red);
-  if (t == 0) a.p2part[(size_t)u * a.nchunks + chunk] = s;
+  const float s_all = block_sum128(valid ? dE : 0.f, red);
+  const float mn = block_min128(cand ? dE : INFINITY, red);
+  const float mx = block_max128(cand ? dE : -INFINITY, red);
+  const float s_de = block_sum128(cand ? dE : 0.f, red);
+  const float s_c = block_sum128(cand ? cosv : 0.f, red);
+  const float s_raw = block_sum128(cand ? vote : 0.f, red);
+  if (t == 0) {
+    float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kP2Stride;
+    p[P2_SUM_DE_ALL] = s_all;
+    p[P2_MIN_DE] = mn;
+    p[P2_MAX_DE] = mx;
+    p[P2_SUM_DE] = s_de;
+    p[P2_SUM_COS] = s_c;
+    p[P2_SUM_RAW] = s_raw;
+  }
 }
 
 template <typename T, int RB>

@@ -1,0 +1,37 @@
+// Launch interface of the persistent tensor-core kernel (tc_pass.cu).
+#pragma once
+
+#include "ecokv_internal.cuh"
+
+namespace ecokv {
+
+constexpr int kTcTilesPerChunk = 8;            // 1024 keys per pass item
+constexpr int kTcChunk = 128 * kTcTilesPerChunk;
+
+struct TcArgs {
+  int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
+  int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
+  int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1
+  int step_items, total_tickets;
+  int p1_stride, ustat_stride;
+  float scale_log2;
+  long long timeout_cycles;
+  const void* Q;
+  float* p1part;
+  float* ustat;
+  float* p2part;
+  float* simp;
+  float* dE;
+  float* cosv;
+  unsigned* sync;                   // [0] ticket, [1] abort, [4+u] pass-1 arrivals, [4+U+u] stats ready
+  unsigned* status;
+};
+
+// Half the MMA N extent (window rows, padded to a multiple of four, plus the
+// mu rows, rounded up to a power of two) for R window rows; 0 when R is too
+// large for this kernel.
+int tc_rows_half(int R);
+size_t tc_smem_bytes();
+cudaError_t launch_tc(const void* K, const TcArgs& args, cudaStream_t st);
+
+}  // namespace ecokv

@@ -15,6 +15,7 @@ LIB_PATH = os.path.join(_HERE, "libecokv.so")
 ECOKV_F32, ECOKV_BF16 = 0, 1
 ECOKV_FLAG_SC_MIXKV_SIGN = 0x1
 ECOKV_FLAG_LAMBDA_OVERRIDE = 0x2
+ECOKV_FLAG_FORCE_SIMT = 0x100
 
 STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED", 3: "ECOKV_ERR_WORKSPACE",
           4: "ECOKV_ERR_CUDA", 5: "ECOKV_ERR_TIMEOUT", 6: "ECOKV_ERR_DEVICE_INDEX"}
