@@ -46,6 +46,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ecokv", "reference"], default="ecokv")
     ap.add_argument("--workload", default="c3_b10")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -245,6 +247,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     w = workload(args.workload)
+    if args.layers:
+        import dataclasses
+        w = dataclasses.replace(w, n_layers=args.layers, name=f"{w.name}_L{args.layers}")
     cores = max(1, min(16, os.cpu_count() or 1))
 
     if args.impl == "reference":
@@ -311,7 +316,7 @@ def main():
 
     # end to end through the public API: pinned host inputs -> device -> pass -> host outputs
     e2e = None
-    if rank == 0 or world > 1:
+    if args.e2e_steps > 0:
         hK = K.cpu().pin_memory()
         hV = V.cpu().pin_memory()
         hQ = Q.cpu().pin_memory()

@@ -2,7 +2,7 @@
 // launches.  Every entry point validates on the host and returns before
 // launching anything when an argument is wrong.
 //
-// Paths.  bf16 inputs with n >= 128 and (h_q/h_kv)*W <= 124 stream K through
+// Paths.  bf16 inputs with n >= 128 and (h_q/h_kv)*W <= 120 stream K through
 // the persistent tensor-core kernel (tc_pass.cu, one launch for both passes);
 // fp32 inputs, other shapes and calls with ECOKV_FLAG_FORCE_SIMT use the
 // CUDA-core passes (score_simt.cu, two launches).  Either way one more launch
@@ -42,6 +42,7 @@ Layout make_layout(const ecokv_params& p, int chunk) {
   L.dE = off;      off += align256(U * L.Tv * 4);
   L.cosv = off;    off += align256(U * L.Tv * 4);
   L.sbuf = off;    off += align256(U * L.Tv * 4);
+  L.norm2 = off;   off += align256(U * (size_t)L.N * 4);
   L.total = off;
   return L;
 }
@@ -64,6 +65,12 @@ static bool use_tensor_path(const ecokv_params& p, ecokv_dtype dt) {
   if (p.n < 128) return false;
   return tc_rows_half((p.h_q / p.h_kv) * p.window) > 0;
 }
+
+static int env_int(const char* name, int dflt, int lo, int hi);
+
+// Keys per tensor-core pass item (128 * tiles; ECOKV_TC_TILES overrides the
+// default of 8 tiles for tuning).
+static int tc_chunk_keys() { return 128 * env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64); }
 
 static int env_int(const char* name, int dflt, int lo, int hi) {
   const char* v = getenv(name);
@@ -140,7 +147,8 @@ static CompactArgs compact_args(const ecokv_params& p, const void* K, const void
 // Both streaming passes on the tensor cores in one launch (after clearing
 // the per-call counters).
 static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
-  const Layout L = make_layout(p, kTcChunk);
+  const int tiles = env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64);
+  const Layout L = make_layout(p, 128 * tiles);
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   TcArgs a{};
   a.U = L.U;
@@ -153,16 +161,18 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.h_kv = p.h_kv;
   a.h_q = p.h_q;
   a.Tv = L.Tv;
-  a.tiles_per_chunk = kTcTilesPerChunk;
+  a.q_rows = p.n_layers * p.h_q * p.window;
+  a.tiles_per_chunk = tiles;
   a.nchunks = L.nchunks;
-  a.lag_p2 = env_int("ECOKV_LAG_P2", 4, 1, 64);
-  a.step_items = 2 * a.nchunks;
-  a.total_tickets = (L.U + a.lag_p2) * a.step_items;
+  a.lag_p2 = env_int("ECOKV_LAG_P2", 8, 1, 64);
+  a.total_tickets = (L.U + a.lag_p2) * 2 * a.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
   a.timeout_cycles = 4000000000LL;  // about 2 s of SM clock per wait
   a.Q = Q;
+  a.K = K;
+  a.norm2 = reinterpret_cast<float*>(ws + L.norm2);
   a.p1part = reinterpret_cast<float*>(ws + L.p1part);
   a.ustat = reinterpret_cast<float*>(ws + L.ustat);
   a.p2part = reinterpret_cast<float*>(ws + L.p2part);
@@ -240,7 +250,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? kTcChunk : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys() : kChunk);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.lambda = lambda;
@@ -298,7 +308,7 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? kTcChunk : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys() : kChunk);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);

@@ -26,6 +26,9 @@ enum : int {
   P2_SUM_COS = 4,     // sum of khat . mu over candidates
   P2_SUM_RAW = 5      // sum of the raw importance vote over candidates
 };
+static_assert(P2_SUM_DE_ALL == 0 && P2_MIN_DE == 1 && P2_MAX_DE == 2 && P2_SUM_DE == 3 && P2_SUM_COS == 4 &&
+                  P2_SUM_RAW == 5,
+              "the pass-2 reductions write the record in this order");
 
 // Device status word (first bytes of the workspace).
 struct DevStatus {
@@ -44,7 +47,7 @@ struct Layout {
   int nchunks;       // ceil(N / chunk)
   int p1_stride;     // floats per (unit, chunk) pass-1 partial: 2R + 2D
   int ustat_stride;  // floats per unit statistics record
-  size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, total;
+  size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2, total;
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
 

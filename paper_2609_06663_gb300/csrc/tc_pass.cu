@@ -9,28 +9,34 @@
 //             key tile as an MN-major operand against [1, w_hi, w_mid, w_lo]
 //             weight rows, w = 1/||k|| split into three bf16 terms).  The last P1 item of a unit folds the partials into the unit
 //             statistics (kbar, mu, per-row log2-sum-exp).
-//   P2(u, c)  pass 2: logits again plus two extra MMA columns holding k . mu
-//             (bf16 hi + lo split of mu), giving the importance vote and the
-//             cosine khat . mu; d_E = ||k - kbar|| (Eq. 1) is taken directly
-//             from the staged key tile in fp32 (the expansion of Sec. 4 cancels
-//             badly when keys sit close to their centroid).
-// Within a schedule step s the list holds P1(s, *) then P2(s - lag_p2, *), so
-// pass 2 of a unit re-reads its keys a few units after pass 1 (from L2, not
-// HBM), and every item depends only on items with smaller tickets: dispatch is
-// deadlock-free without co-residency.  Pass 2 leaves per-candidate arrays and
-// per-chunk partial sums; finalisation, selection and the gather of the kept
-// rows run in the next launch (finalize_select.cu).
+//   P2(u, c)  pass 2: logits again plus five extra MMA columns holding k . kbar
+//             (kbar split into three bf16 terms) and k . mu (two terms), giving
+//             the importance vote, the cosine khat . mu, and d_E (Eq. 1) by the
+//             expansion of Sec. 4 from ||k||^2 (stored by pass 1).  Where that
+//             expansion cancels (d_E^2 below 2^-6 of ||k||^2 + ||kbar||^2, keys
+//             close to their centroid) the key is recomputed directly from its
+//             row in global memory.
+// Work is a global, ticket-ordered list of items.  Within a schedule step s
+// the list holds P1(s, *) then P2(s - lag_p2, *), so pass 2 of a unit re-reads
+// its keys a few units after pass 1 (from L2 when the keys streamed in
+// between fit), and every item depends only on items with smaller tickets:
+// dispatch is deadlock-free without co-residency.  Pass 2 leaves
+// per-candidate arrays and per-chunk partial sums; finalisation, selection
+// and the gather of the kept rows run in the next launch (finalize_select.cu).
 //
-// Warp roles (320 threads, one CTA per SM): warp 0 takes tickets, resolves
-// dependencies (bounded spins on gpu-scope flags), builds the MMA B operand
-// (window queries, plus the kbar / mu rows for pass 2) and issues TMA loads of
-// 32 KB key tiles into a 4-stage ring; warp 1 issues tcgen05 MMAs into a
-// double-buffered TMEM accumulator; warps 2-9 are the epilogue (one key per
-// TMEM lane, window rows split in two halves).  Every mbarrier wait and spin
+// Warp roles (384 threads, one CTA per SM): warp 0 takes tickets, resolves
+// dependencies (bounded spins on gpu-scope flags), loads the window queries
+// (TMA) and the unit statistics (bulk copy) and issues TMA loads of 32 KB key
+// tiles into a 4-stage ring; warp 1 issues the tcgen05 MMAs into up to four
+// TMEM accumulators (plus two for the sums); warps 2-3 (key warps) compute
+// the key norms and the sum weights of each pass-1 tile as soon as it lands,
+// so that a ring stage is freed without waiting for the softmax; warps 4-11
+// are the epilogue (one key per TMEM lane, window rows split in two halves).  Every mbarrier wait and spin
 // is bounded: on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
 // gpu-wide abort flag, drains its own copies and MMAs, frees TMEM and exits.
 
 #include <cuda.h>
+#include <stddef.h>
 
 #include "finalize_select.cuh"
 #include "ptx.cuh"
@@ -41,11 +47,11 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kStages = 4;
 constexpr int kIQ = 2;
 constexpr int kTile = 128;
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
 constexpr int kEpi = 256;
+constexpr int kEpiWarp0 = 4;          // first epilogue warp
 constexpr int kNPMax = 128;
 constexpr uint32_t kTileBytes = kTile * kD * 2;
 constexpr uint32_t kTmemCols = 512;
@@ -54,31 +60,41 @@ constexpr uint32_t kEpiBar = 1;
 
 enum : int { kP1 = 0, kP2 = 1, kExit = 3 };
 
-struct ItemDesc {
+constexpr int kUstatMax = (2 * kD + 2 + kNPMax + 3) & ~3;  // floats of a unit statistics record
+
+struct __align__(16) ItemDesc {
   int type, u, chunk, part, i0, ntiles;
-  float lse[kNPMax];
-  float kbar[kD];
+  int pad[2];
+  float ust[kUstatMax];  // pass 2: copy of the unit statistics record (kbar, mu, norms, log2-LSE)
 };
 
+// Shared memory of the kernel instance with RH window rows per half: the
+// query buffers take just 2 * RH rows, which leaves room for a fifth key-tile
+// stage unless RH = 64.
+template <int RH>
 struct __align__(1024) Smem {
-  uint8_t ktile[kStages][kTileBytes];   // 2 boxes [128 keys x 64 d], 128-byte swizzle
-  uint8_t qbuf[kIQ][kNPMax * 256];      // B operand, 2 boxes [NP rows x 64 d]
-  uint8_t wbuf[kStages][4096];          // sum weights: 2 boxes [16 rows x 64 keys]; rows 1, w_hi, w_mid, w_lo
+  static constexpr int kS = RH >= 64 ? 4 : 5;  // key-tile stages
+  static constexpr int kQB = 2 * RH * 256;      // bytes of one query buffer (2 boxes of 2*RH rows)
+  uint8_t ktile[kS][kTileBytes];                // 2 boxes [128 keys x 64 d], 128-byte swizzle
+  uint8_t qbuf[kIQ][kQB < 1024 ? 1024 : kQB];   // B operand, 2 boxes [NP rows x 64 d]
+  uint8_t wbuf[kS][4096];                       // sum weights: 2 boxes [16 rows x 64 keys]; rows 1, w_hi, w_mid, w_lo
   ItemDesc desc[kIQ];
-  float xch[2][2][kTile];               // [tile parity][row half][key]
-  float xd2[2][2][kTile];               // squared distance to kbar, per half
-  float xn2[2][2][kTile];               // squared key norm, per half
-  float red[8][64][2];                  // [epilogue warp][row][max, sum]
+  float xch[2][2][kTile];                       // [tile parity][row half][key]
+  float red[8][RH][2];                          // [epilogue warp][row][max, sum]
+  float red6[8][8];                             // [epilogue warp][pass-2 partial]
   float shf[64];
-  uint64_t full[kStages], empty[kStages], wready[kStages];
-  uint64_t item_full[kIQ], item_empty[kIQ];
-  uint64_t tmem_full[2], tmem_empty[2];
-  uint64_t sigma_full, sigma_empty, drain;
+  uint64_t full[kS], empty[kS], wready[kS];
+  uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
+  uint64_t tmem_full[4], tmem_empty[4];
+  uint64_t sigma_full[2], sigma_empty[2], drain;
   uint32_t tmem_base;
   int flag_last;
 };
 
-static_assert(sizeof(Smem) + 1024 <= 232448, "shared-memory plan exceeds the 227 KB per-CTA limit");
+static_assert(sizeof(Smem<8>) + 1024 <= 232448 && sizeof(Smem<16>) + 1024 <= 232448 &&
+                  sizeof(Smem<32>) + 1024 <= 232448 && sizeof(Smem<64>) + 1024 <= 232448,
+              "shared-memory plan exceeds the 227 KB per-CTA limit");
+static_assert(sizeof(ItemDesc) % 16 == 0 && offsetof(ItemDesc, ust) % 16 == 0, "bulk-copy target alignment");
 
 struct EpiSync {
   __device__ __forceinline__ static void sync() { named_bar_sync(kEpiBar, kEpi); }
@@ -111,29 +127,17 @@ __device__ bool wait_bar(uint64_t* bar, uint32_t parity, const TcArgs& a, unsign
   }
 }
 
-// Bounded spin on a gpu-scope flag written by another CTA.
-__device__ bool wait_flag(const unsigned* f, const TcArgs& a, unsigned where) {
-  const long long t0 = clock64();
-  while (ld_acquire(f) == 0u) {
-    if (aborted(a)) return false;
-    if (clock64() - t0 > a.timeout_cycles) {
-      raise_abort(a, ECOKV_ERR_TIMEOUT, where);
-      return false;
-    }
-    __nanosleep(256);
-  }
-  return true;
-}
-
 struct Item {
   int type, u, chunk, part;
   bool valid;
 };
 
+// Item of a ticket: step s = ticket / (2 * nchunks) holds the P1 items of unit
+// s and then the P2 items of unit s - lag_p2 (invalid outside [0, U)).
 __device__ Item decode(int ticket, const TcArgs& a) {
   Item it{kExit, 0, 0, 0, true};
   if (ticket >= a.total_tickets) return it;
-  const int s = ticket / a.step_items, slot = ticket % a.step_items;
+  const int s = ticket / (2 * a.nchunks), slot = ticket - s * 2 * a.nchunks;
   if (slot < a.nchunks) {
     it.type = kP1;
     it.u = s;
@@ -147,6 +151,20 @@ __device__ Item decode(int ticket, const TcArgs& a) {
   return it;
 }
 
+// Bounded spin on a gpu-scope flag written by another CTA.
+__device__ bool wait_flag(const unsigned* f, const TcArgs& a, unsigned where) {
+  const long long t0 = clock64();
+  while (ld_acquire(f) == 0u) {
+    if (aborted(a)) return false;
+    if (clock64() - t0 > a.timeout_cycles) {
+      raise_abort(a, ECOKV_ERR_TIMEOUT, where);
+      return false;
+    }
+    __nanosleep(128);
+  }
+  return true;
+}
+
 __device__ __forceinline__ uint32_t sw128(int row, int chunk16) {
   return (uint32_t)(row * 128 + ((chunk16 ^ (row & 7)) << 4));
 }
@@ -156,76 +174,91 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// B operand of one item in the 128-byte-swizzled K-major layout: rows 0..R-1
-// are the group's window queries; for pass 2, rows R4 and R4+1 hold mu_hi and
-// mu_lo; every other row is zero.  Run by the 32 lanes of warp 0.
-__device__ void build_qbuf(uint8_t* qb, const TcArgs& a, const Item& it, int lane) {
-  const int layer = it.u / a.h_kv, head = it.u % a.h_kv;
-  const uint4* Qu = reinterpret_cast<const uint4*>(a.Q) + ((size_t)layer * a.h_q + (size_t)head * a.g) * a.W * 16;
-  const float* us = a.ustat + (size_t)it.u * a.ustat_stride;
-  for (int e = lane; e < a.NP * 16; e += 32) {
-    const int r = e >> 4, j = e & 15;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (r < a.R) {
-      val = __ldg(Qu + (size_t)r * 16 + j);
-    } else if (it.type == kP2 && r >= a.R4 && r < a.R4 + 2) {
-      const int which = r - a.R4;
-      const float* src = us + ustat_mu() + j * 8;
-      float x[8], o[8];
+// Pass-2 rows of the B operand (128-byte-swizzled, K-major): rows R4..R4+2
+// hold kbar split into three bf16 terms (hi, mid, lo), rows R4+3, R4+4 hold
+// mu_hi and mu_lo, all from the unit statistics copy; the window queries in
+// rows 0..R-1 arrive by TMA.  Run by the 32 lanes of warp 0.
+__device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, const float* ust, int lane) {
+  for (int e = lane; e < 5 * 16; e += 32) {
+    const int which = e >> 4, j = e & 15;
+    const float* src = ust + (which < 3 ? ustat_kbar() : ustat_mu()) + j * 8;
+    const int term = which < 3 ? which : which - 3;  // 0 = hi, 1 = mid / lo, 2 = lo
+    float o[8];
 #pragma unroll
-      for (int t = 0; t < 8; ++t) {
-        x[t] = __ldcg(src + t);
-        const float hi = __bfloat162float(__float2bfloat16_rn(x[t]));
-        o[t] = (which & 1) ? (x[t] - hi) : hi;
-      }
-      val = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
-                       pack_bf16x2(o[6], o[7]));
+    for (int t = 0; t < 8; ++t) {
+      const float x = src[t];
+      const float hi = __bfloat162float(__float2bfloat16_rn(x));
+      const float r1 = x - hi;
+      const float mid = __bfloat162float(__float2bfloat16_rn(r1));
+      o[t] = term == 0 ? hi : (which < 3 ? (term == 1 ? mid : r1 - mid) : r1);
     }
-    *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(r, j & 7)) = val;
+    const uint4 val = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                                 pack_bf16x2(o[6], o[7]));
+    *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(a.R4 + which, j & 7)) = val;
   }
 }
 
-__device__ __forceinline__ float warp_max_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-__device__ __forceinline__ float warp_sum_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 // Fold every chunk's pass-1 partials of unit u into its statistics record.
-__device__ void unit_reduce(const TcArgs& a, int u, Smem& s, int tid) {
+// Threads [0, R) take one window row each (chunk maxima, then the rescaled
+// exp-sums), threads [128, 256) one key dimension each (sums of k and of
+// k/||k||); loads go out in batches of 16 so the L2 latency is paid a few
+// times per unit rather than once per chunk.
+__device__ void unit_reduce(const TcArgs& a, int u, float* shf, int tid) {
   __threadfence();
+  constexpr int kB = 16;
   const float* base = a.p1part + (size_t)u * a.nchunks * a.p1_stride;
   float* us = a.ustat + (size_t)u * a.ustat_stride;
+  const int nch = a.nchunks;
   float kb = 0.f, mu = 0.f;
-  if (tid < kD) {
+  if (tid < a.R) {
+    const int r = tid;
+    float M = -INFINITY;
+    for (int c0 = 0; c0 < nch; c0 += kB) {
+      float mv[kB];
+#pragma unroll
+      for (int j = 0; j < kB; ++j) mv[j] = c0 + j < nch ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + r) : -INFINITY;
+#pragma unroll
+      for (int j = 0; j < kB; ++j) M = fmaxf(M, mv[j]);
+    }
+    float Z = 0.f;
+    for (int c0 = 0; c0 < nch; c0 += kB) {
+      float mv[kB], zv[kB];
+#pragma unroll
+      for (int j = 0; j < kB; ++j) {
+        const bool in = c0 + j < nch;
+        mv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + r) : -INFINITY;
+        zv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + a.R + r) : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < kB; ++j)
+        if (mv[j] != -INFINITY) Z += zv[j] * ex2(mv[j] - M);
+    }
+    us[ustat_lse() + r] = M + log2f(Z);
+  } else if (tid >= 128) {
+    const int dd = tid - 128;
     float sk = 0.f, skh = 0.f;
-    for (int c = 0; c < a.nchunks; ++c) {
-      sk += __ldcg(base + (size_t)c * a.p1_stride + 2 * a.R + tid);
-      skh += __ldcg(base + (size_t)c * a.p1_stride + 2 * a.R + kD + tid);
+    for (int c0 = 0; c0 < nch; c0 += kB) {
+      float kv[kB], hv[kB];
+#pragma unroll
+      for (int j = 0; j < kB; ++j) {
+        const bool in = c0 + j < nch;
+        kv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + 2 * a.R + dd) : 0.f;
+        hv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + 2 * a.R + kD + dd) : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < kB; ++j) {
+        sk += kv[j];
+        skh += hv[j];
+      }
     }
     const float inv_n = 1.f / (float)a.N;
     kb = sk * inv_n;
     mu = skh * inv_n;
-    us[ustat_kbar() + tid] = kb;
-    us[ustat_mu() + tid] = mu;
+    us[ustat_kbar() + dd] = kb;
+    us[ustat_mu() + dd] = mu;
   }
-  for (int row = tid; row < a.R; row += kEpi) {
-    float M = -INFINITY;
-    for (int c = 0; c < a.nchunks; ++c) M = fmaxf(M, __ldcg(base + (size_t)c * a.p1_stride + row));
-    float Z = 0.f;
-    for (int c = 0; c < a.nchunks; ++c) {
-      const float m = __ldcg(base + (size_t)c * a.p1_stride + row);
-      if (m != -INFINITY) Z += __ldcg(base + (size_t)c * a.p1_stride + a.R + row) * exp2f(m - M);
-    }
-    us[ustat_lse() + row] = M + log2f(Z);
-  }
-  const float ksq = group_reduce<Op::Sum, EpiSync>(kb * kb, s.shf, tid, kEpi);
-  const float msq = group_reduce<Op::Sum, EpiSync>(mu * mu, s.shf, tid, kEpi);
+  const float ksq = group_reduce<Op::Sum, EpiSync>(kb * kb, shf, tid, kEpi);
+  const float msq = group_reduce<Op::Sum, EpiSync>(mu * mu, shf, tid, kEpi);
   if (tid == 0) {
     us[ustat_ksq()] = ksq;
     us[ustat_musq()] = msq;
@@ -233,27 +266,34 @@ __device__ void unit_reduce(const TcArgs& a, int u, Smem& s, int tid) {
 }
 
 template <int RH>
-__global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_constant__ CUtensorMap tmK, TcArgs a) {
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_evict_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  Smem& s = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  using SM = Smem<RH>;
+  constexpr int kStages = SM::kS;
+  SM& s = *reinterpret_cast<SM*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nbuf_log = a.NP <= 64 ? 2 : 1;  // 4 or 2 TMEM accumulators of NP columns (<= 256 columns)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], 9);
-      mbar_init(&s.wready[i], 8);
+      mbar_init(&s.empty[i], 3);   // 2 key warps + MMA commit
+      mbar_init(&s.wready[i], 2);  // 2 key warps
     }
     for (int i = 0; i < kIQ; ++i) {
       mbar_init(&s.item_full[i], 1);
-      mbar_init(&s.item_empty[i], 2);
+      mbar_init(&s.item_empty[i], 11);  // MMA commit + 8 epilogue warps + 2 key warps
+      mbar_init(&s.qfull[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 4; ++i) {
       mbar_init(&s.tmem_full[i], 1);
       mbar_init(&s.tmem_empty[i], 8);
     }
-    mbar_init(&s.sigma_full, 1);
-    mbar_init(&s.sigma_empty, 4);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.sigma_full[i], 1);
+      mbar_init(&s.sigma_empty[i], 4);
+    }
     mbar_init(&s.drain, 1);
     fence_mbar_init();
   }
@@ -268,7 +308,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
     tmem_alloc(&s.tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  if (warp == 0 && lane == 0) tma_prefetch_desc(&tmK);
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmQ);
+  }
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
@@ -283,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
     uint32_t used_bits = 0u, par_bits = 0u;  // per stage: loaded at least once / parity of loads
     for (int seq = 0; ok;) {
       int ticket = 0;
-      if (lane == 0) ticket = atomicAdd(a.sync, 1u);
+      if (lane == 0) ticket = (int)atomicAdd(a.sync, 1u);
       ticket = __shfl_sync(0xffffffffu, ticket, 0);
       const Item it = decode(ticket, a);
       if (!it.valid) continue;
@@ -307,12 +350,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
         d.ntiles = ntiles;
       }
       if (it.type == kP1 || it.type == kP2) {
-        build_qbuf(s.qbuf[slot], a, it, lane);
-        if (it.type == kP2) {
-          const float* us = a.ustat + (size_t)it.u * a.ustat_stride;
-          for (int r = lane; r < a.R; r += 32) d.lse[r] = __ldcg(us + ustat_lse() + r);
-          for (int c = lane; c < kD; c += 32) d.kbar[c] = __ldcg(us + ustat_kbar() + c);
+        // window queries by TMA (swizzled in flight); pass 2 also copies the
+        // unit statistics record
+        const uint32_t ust_bytes = (uint32_t)a.ustat_stride * 4u;
+        if (lane == 0) {
+          const int layer = it.u / a.h_kv, head = it.u % a.h_kv;
+          const int qrow = (layer * a.h_q + head * a.g) * a.W;
+          mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u + (it.type == kP2 ? ust_bytes : 0u));
+          tma_load_2d(s.qbuf[slot], &tmQ, &s.qfull[slot], 0, qrow);
+          tma_load_2d(s.qbuf[slot] + a.NP * 128, &tmQ, &s.qfull[slot], 64, qrow);
+          if (it.type == kP2) bulk_load(d.ust, a.ustat + (size_t)it.u * a.ustat_stride, ust_bytes, &s.qfull[slot]);
+          ok = wait_bar(&s.qfull[slot], qphase, a, 16u);
         }
+        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        if (!ok) break;
+        if (it.type == kP2) build_stat_rows(s.qbuf[slot], a, d.ust, lane);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -363,9 +415,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
         const ItemDesc& d = s.desc[slot];
         const int type = d.type, ntiles = d.ntiles;
         if (type == kExit) break;
+        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
+        tc_fence_after();
         const uint32_t qb = smem_u32(s.qbuf[slot]);
         for (int t = 0; t < ntiles; ++t) {
-          const uint32_t b = tcount & 1u, tph = (tcount >> 1) & 1u;
+          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.full[stage], sphase, a, 6u))) break;
           if (!(ok = wait_bar(&s.tmem_empty[b], tph ^ 1u, a, 7u))) break;
           tc_fence_after();
@@ -374,13 +428,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
           for (int kk = 0; kk < 8; ++kk) {
             const uint64_t ad = smem_desc(kt + (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32, 16, 1024, 2);
             const uint64_t bd = smem_desc(qb + (kk >> 2) * (a.NP * 128) + (kk & 3) * 32, 16, 1024, 2);
-            mma_bf16(tmem + b * 128u, ad, bd, idesc_l, kk > 0 ? 1u : 0u);
+            mma_bf16(tmem + b * (uint32_t)a.NP, ad, bd, idesc_l, kk > 0 ? 1u : 0u);
           }
           mma_commit(&s.tmem_full[b]);
           if (type == kP1) {
             if (!(ok = wait_bar(&s.wready[stage], (wpar >> stage) & 1u, a, 8u))) break;
             wpar ^= 1u << stage;
-            if (t == 0 && !(ok = wait_bar(&s.sigma_empty, (sigcount & 1u) ^ 1u, a, 9u))) break;
+            const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+            if (t == 0 && !(ok = wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u))) break;
             tc_fence_after();
             const uint32_t wb = smem_u32(s.wbuf[stage]);
 #pragma unroll
@@ -388,12 +443,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
               // A = key tile viewed MN-major (d contiguous): 16 keys per step
               const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
               const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
-              mma_bf16(tmem + kSigmaCol, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
+              mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
             }
           }
           mma_commit(&s.empty[stage]);
           if (type == kP1 && t == ntiles - 1) {
-            mma_commit(&s.sigma_full);
+            mma_commit(&s.sigma_full[sigcount & 1u]);
             ++sigcount;
           }
           ++tcount;
@@ -412,15 +467,101 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
         }
       }
     }
-  } else {
-    // ------------------------------------------------ epilogue (warps 2..9)
-    const int e = warp - 2, q = warp & 3, h = e >> 2;
-    const int kk = 32 * q + lane;  // key row within a tile = TMEM lane
-    const int tid = threadIdx.x - 64;
-    const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+  } else if (warp < kEpiWarp0) {
+    // ------------------------------------------------ key warps (2..3)
+    const int tk = threadIdx.x - 64;  // 0..63: keys tk and tk + 64 of each tile
     int stage = 0;
-    uint32_t sphase = 0, tcount = 0, sigcount = 0;
+    uint32_t sphase = 0;
     for (int seq = 0; ok; ++seq) {
+      const int slot = seq % kIQ;
+      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+      if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 20u))) break;
+      const ItemDesc& d = s.desc[slot];
+      const int type = d.type, ntiles = d.ntiles, i0 = d.i0, u = d.u;
+      if (type == kExit) break;
+      for (int t = 0; t < ntiles && ok; ++t) {
+        if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
+        if (type == kP1) {
+          // squared norms, the sum weights w = 1/||k|| (three bf16 terms) and
+          // the norms for pass 2
+#pragma unroll
+          for (int q2 = 0; q2 < 2; ++q2) {
+            const int kk = tk + 64 * q2;
+            float n2p[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int hb = 0; hb < 2; ++hb) {
+              const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
+#pragma unroll
+              for (int c = 0; c < 8; ++c) {
+                const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
+                const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int t2 = 0; t2 < 4; ++t2) {
+                  const float lo = __uint_as_float(w4[t2] << 16), hi = __uint_as_float(w4[t2] & 0xffff0000u);
+                  n2p[t2] = fmaf(lo, lo, n2p[t2]);
+                  n2p[t2] = fmaf(hi, hi, n2p[t2]);
+                }
+              }
+            }
+            const float n2 = (n2p[0] + n2p[1]) + (n2p[2] + n2p[3]);
+            const int i = i0 + t * kTile + kk;
+            const bool valid = i < a.N;
+            if (valid) a.norm2[(size_t)u * a.N + i] = n2;
+            const float w = valid ? 1.f / fmaxf(sqrtf(n2), 1e-12f) : 0.f;
+            const __nv_bfloat16 whi = __float2bfloat16_rn(w);
+            const float r1 = w - __bfloat162float(whi);
+            const __nv_bfloat16 wmid = __float2bfloat16_rn(r1);
+            const __nv_bfloat16 wlo = __float2bfloat16_rn(r1 - __bfloat162float(wmid));
+            uint8_t* base = s.wbuf[stage] + (kk >> 6) * 2048 + (kk & 7) * 2;
+            const int j = (kk & 63) >> 3;
+            *reinterpret_cast<__nv_bfloat16*>(base + sw128(1, j)) = whi;
+            *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
+            *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;
+          }
+          __threadfence();  // key norms visible before the unit's pass-1 arrival count
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.wready[stage]);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
+        if (++stage == kStages) {
+          stage = 0;
+          sphase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 4..11)
+    const int e = warp - kEpiWarp0, q = warp & 3, h = e >> 2;
+    const int kk = 32 * q + lane;  // key row within a tile = TMEM lane
+    const int tid = threadIdx.x - 32 * kEpiWarp0;
+    const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+    uint32_t tcount = 0, sigcount = 0;
+    int pending_u = -1;        // unit of the last pass-1 arrival still to resolve
+    unsigned pending_old = 0;  // what the arrival counter held before it (thread 0)
+    for (int seq = 0; ok; ++seq) {
+      if (pending_u >= 0) {
+        // the pass-1 arrival of the previous item: the last of its unit folds
+        // the chunk partials into the unit statistics
+        if (tid == 0) s.flag_last = pending_old == (unsigned)(a.nchunks - 1);
+        named_bar_sync(kEpiBar, kEpi);
+        const bool last = s.flag_last != 0;
+        named_bar_sync(kEpiBar, kEpi);
+        if (last) {
+          unit_reduce(a, pending_u, s.shf, tid);
+          __threadfence();
+          named_bar_sync(kEpiBar, kEpi);
+          if (tid == 0) {
+            __threadfence();
+            st_release(a.sync + 4 + a.U + pending_u, 1u);
+          }
+        }
+        pending_u = -1;
+      }
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
       if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 10u))) break;
@@ -440,194 +581,158 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
           const int it0 = i0 + t * kTile;
           const int i = it0 + kk;
           const bool valid = i < a.N;
-          // key norm: this half of the row, exchanged with the other half
-          if (!(ok = wait_bar(&s.full[stage], sphase, a, 11u))) break;
-          const uint8_t* row = s.ktile[stage] + h * (kTileBytes / 2) + kk * 128;
-          float n2h = 0.f;
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
-            const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-            float p = 0.f;
-#pragma unroll
-            for (int t2 = 0; t2 < 4; ++t2) {
-              const float lo = __uint_as_float(w4[t2] << 16), hi = __uint_as_float(w4[t2] & 0xffff0000u);
-              p = fmaf(lo, lo, p);
-              p = fmaf(hi, hi, p);
-            }
-            n2h += p;
-          }
-          s.xch[t & 1][h][kk] = n2h;
-          named_bar_sync(kEpiBar, kEpi);
-          const float n2 = s.xch[t & 1][0][kk] + s.xch[t & 1][1][kk];
-          const float w = valid ? 1.f / fmaxf(sqrtf(n2), 1e-12f) : 0.f;
-          {
-            // w = w_hi + w_mid + w_lo in bf16 (about 24 significant bits)
-            const __nv_bfloat16 whi = __float2bfloat16_rn(w);
-            const float r1 = w - __bfloat162float(whi);
-            const __nv_bfloat16 wmid = __float2bfloat16_rn(r1);
-            const __nv_bfloat16 wlo = __float2bfloat16_rn(r1 - __bfloat162float(wmid));
-            uint8_t* base = s.wbuf[stage] + (kk >> 6) * 2048 + (kk & 7) * 2;
-            const int j = (kk & 63) >> 3;
-            if (h == 0) {
-              *reinterpret_cast<__nv_bfloat16*>(base + sw128(1, j)) = whi;
-            } else {
-              *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
-              *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;
-            }
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            mbar_arrive(&s.wready[stage]);
-            mbar_arrive(&s.empty[stage]);  // done reading the key tile
-          }
-
-          // window logits of this key
-          const uint32_t b = tcount & 1u, tph = (tcount >> 1) & 1u;
+          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 12u))) break;
           tc_fence_after();
           uint32_t r[RH];
-          tmem_ld<RH>(tl + b * 128u + (uint32_t)(h * RH), r);
+          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), r);
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
-          const bool all_vis = it0 + kTile - 1 <= a.N - a.W;
+          // online softmax partials, branch-free: re-base the running sum only
+          // when a logit exceeds the running reference by more than 2^20
+          if (it0 + kTile - 1 <= a.N - a.W) {
+            // every key of the tile is visible to every window row
 #pragma unroll
-          for (int c = 0; c < RH; ++c) {
-            const int rowi = h * RH + c;
-            if (rowi < a.R) {
-              const bool vis = all_vis || (valid && i <= a.N - a.W + (rowi % a.W));
-              if (vis) {
-                const float x = __uint_as_float(r[c]) * a.scale_log2;
-                const float dlt = x - m[c];
-                if (dlt > 20.f) {
-                  z[c] = fmaf(z[c], exp2f(-dlt), 1.f);
-                  m[c] = x;
-                } else {
-                  z[c] += exp2f(dlt);
-                }
-              }
+            for (int c = 0; c < RH; ++c) {
+              const float x = __uint_as_float(r[c]) * a.scale_log2;
+              const float dlt = (h * RH + c < a.R) ? x - m[c] : -INFINITY;
+              const bool up = dlt > 20.f;
+              const float ee = ex2(up ? -dlt : dlt);
+              z[c] = up ? fmaf(z[c], ee, 1.f) : z[c] + ee;
+              m[c] = up ? x : m[c];
+            }
+          } else {
+            // last tiles of the unit: window row j sees keys i <= N - W + j,
+            // and keys past N do not exist
+            const int vis_from = i - (a.N - a.W);  // row j sees key i iff j >= vis_from
+            int j = (h * RH) % a.W;
+#pragma unroll
+            for (int c = 0; c < RH; ++c) {
+              const bool vis = (h * RH + c < a.R) && valid && j >= vis_from;
+              if (++j == a.W) j = 0;
+              const float x = __uint_as_float(r[c]) * a.scale_log2;
+              const float dlt = vis ? x - m[c] : -INFINITY;
+              const bool up = dlt > 20.f;
+              const float ee = ex2(up ? -dlt : dlt);
+              z[c] = up ? fmaf(z[c], ee, 1.f) : z[c] + ee;
+              m[c] = up ? x : m[c];
             }
           }
           ++tcount;
-          if (++stage == kStages) {
-            stage = 0;
-            sphase ^= 1u;
-          }
         }
         if (!ok) break;
-        // item end: per-row (max, sum) over the 32 keys of the warp
+        // item end: per-row (max, sum) over the 32 keys of the warp, step-major
+        // so that the RH rows' shuffles overlap
+        float M[RH];
 #pragma unroll
-        for (int c = 0; c < RH; ++c) {
-          const float M = warp_max_f(m[c]);
-          const float zz = (m[c] == -INFINITY) ? 0.f : z[c] * exp2f(m[c] - M);
-          const float Z = warp_sum_f(zz);
-          if (lane == 0) {
-            s.red[e][c][0] = M;
-            s.red[e][c][1] = Z;
+        for (int c = 0; c < RH; ++c) M[c] = m[c];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+          for (int c = 0; c < RH; ++c) M[c] = fmaxf(M[c], __shfl_xor_sync(0xffffffffu, M[c], o));
+        }
+#pragma unroll
+        for (int c = 0; c < RH; ++c) z[c] = (m[c] == -INFINITY) ? 0.f : z[c] * ex2(m[c] - M[c]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+          for (int c = 0; c < RH; ++c) z[c] += __shfl_xor_sync(0xffffffffu, z[c], o);
+        }
+        if (lane == 0) {
+#pragma unroll
+          for (int c = 0; c < RH; ++c) {
+            s.red[e][c][0] = M[c];
+            s.red[e][c][1] = z[c];
           }
         }
         named_bar_sync(kEpiBar, kEpi);
         float* part = a.p1part + ((size_t)u * a.nchunks + chunk) * a.p1_stride;
         if (tid < a.R) {
           const int hh = tid / RH, c = tid % RH;
-          float M = -INFINITY;
+          float Mx = -INFINITY;
 #pragma unroll
-          for (int w4 = 0; w4 < 4; ++w4) M = fmaxf(M, s.red[4 * hh + w4][c][0]);
+          for (int w4 = 0; w4 < 4; ++w4) Mx = fmaxf(Mx, s.red[4 * hh + w4][c][0]);
           float Z = 0.f;
 #pragma unroll
           for (int w4 = 0; w4 < 4; ++w4) {
             const float mm = s.red[4 * hh + w4][c][0];
-            if (mm != -INFINITY) Z += s.red[4 * hh + w4][c][1] * exp2f(mm - M);
+            if (mm != -INFINITY) Z += s.red[4 * hh + w4][c][1] * ex2(mm - Mx);
           }
-          part[tid] = M;
+          part[tid] = Mx;
           part[a.R + tid] = Z;
         }
         // chunk sums of k and k/||k|| from the weight MMA (TMEM lane = dimension)
         if (h == 0) {
-          if (!(ok = wait_bar(&s.sigma_full, sigcount & 1u, a, 13u))) break;
+          const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+          if (!(ok = wait_bar(&s.sigma_full[sb], sph, a, 13u))) break;
           tc_fence_after();
           uint32_t v[4];
-          tmem_ld_x4(tl + kSigmaCol, v);
+          tmem_ld_x4(tl + kSigmaCol + 16u * sb, v);
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&s.sigma_empty);
+          if (lane == 0) mbar_arrive(&s.sigma_empty[sb]);
           part[2 * a.R + kk] = __uint_as_float(v[0]);
           part[2 * a.R + kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
         }
         ++sigcount;
-        __threadfence();  // this thread's partials and key norms before the arrival count
+        __threadfence();  // this thread's partials before the arrival count
         named_bar_sync(kEpiBar, kEpi);
-        if (tid == 0) {
-          __threadfence();
-          const unsigned old = atom_add_acq_rel(a.sync + 4 + u, 1u);
-          s.flag_last = old == (unsigned)(a.nchunks - 1);
-        }
-        named_bar_sync(kEpiBar, kEpi);
-        if (s.flag_last) {
-          unit_reduce(a, u, s, tid);
-          __threadfence();
-          named_bar_sync(kEpiBar, kEpi);
-          if (tid == 0) {
-            __threadfence();
-            st_release(a.sync + 4 + a.U + u, 1u);
-          }
-        }
-      } else if (type == kP2) {
+        if (tid == 0) pending_old = atom_add_acq_rel(a.sync + 4 + u, 1u);  // resolved at the next loop top
+        pending_u = u;
+      } else {  // kP2
+        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 18u))) break;  // statistics copy landed
+        const float* lse = d.ust + ustat_lse();
+        const float* kbv = d.ust + ustat_kbar();
+        const float ksq = d.ust[ustat_ksq()];
         float s_all = 0.f, mn = INFINITY, mx = -INFINITY, s_de = 0.f, s_c = 0.f, s_raw = 0.f;
-        const float* kb = d.kbar + h * 64;
         for (int t = 0; t < ntiles && ok; ++t) {
           const int i = i0 + t * kTile + kk;
           const bool valid = i < a.N;
-          // distance to the centroid and squared norm over this half's 64 dims
-          if (!(ok = wait_bar(&s.full[stage], sphase, a, 15u))) break;
-          const uint8_t* row = s.ktile[stage] + h * (kTileBytes / 2) + kk * 128;
-          float d2h = 0.f, n2h = 0.f;
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
-            const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-            for (int t2 = 0; t2 < 4; ++t2) {
-              const float lo = __uint_as_float(w4[t2] << 16), hi = __uint_as_float(w4[t2] & 0xffff0000u);
-              const float dl = lo - kb[c * 8 + 2 * t2], dh = hi - kb[c * 8 + 2 * t2 + 1];
-              d2h = fmaf(dl, dl, d2h);
-              d2h = fmaf(dh, dh, d2h);
-              n2h = fmaf(lo, lo, n2h);
-              n2h = fmaf(hi, hi, n2h);
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.empty[stage]);  // done reading the key tile
-          const uint32_t b = tcount & 1u, tph = (tcount >> 1) & 1u;
+          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 14u))) break;
           tc_fence_after();
-          uint32_t r[RH], st4[4];
-          tmem_ld<RH>(tl + b * 128u + (uint32_t)(h * RH), r);
-          if (h == 0) tmem_ld_x4(tl + b * 128u + (uint32_t)a.R4, st4);
+          uint32_t r[RH], st[8];
+          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), r);
+          if (h == 0) tmem_ld_x8(tl + b * (uint32_t)a.NP + (uint32_t)a.R4, st);
+          const float n2 = (h == 0 && valid) ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
-          float vote = 0.f;
+          float vp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < RH; ++c) {
             const int rowi = h * RH + c;
-            if (rowi < a.R) vote += exp2f(fmaf(__uint_as_float(r[c]), a.scale_log2, -d.lse[rowi]));
+            if (rowi < a.R) vp[c & 3] += ex2(fmaf(__uint_as_float(r[c]), a.scale_log2, -lse[rowi]));
           }
-          s.xch[t & 1][h][kk] = vote;
-          s.xd2[t & 1][h][kk] = d2h;
-          s.xn2[t & 1][h][kk] = n2h;
+          s.xch[tcount & 1u][h][kk] = (vp[0] + vp[1]) + (vp[2] + vp[3]);
           named_bar_sync(kEpiBar, kEpi);
           if (h == 0 && valid) {
-            const float v = s.xch[t & 1][0][kk] + s.xch[t & 1][1][kk];
-            const float d2 = s.xd2[t & 1][0][kk] + s.xd2[t & 1][1][kk];
-            const float n2 = s.xn2[t & 1][0][kk] + s.xn2[t & 1][1][kk];
-            const float kmu = __uint_as_float(st4[0]) + __uint_as_float(st4[1]);
-            const float dEv = sqrtf(d2);
+            const float v = s.xch[tcount & 1u][0][kk] + s.xch[tcount & 1u][1][kk];
+            const float kkb = (__uint_as_float(st[0]) + __uint_as_float(st[1])) + __uint_as_float(st[2]);
+            const float kmu = __uint_as_float(st[3]) + __uint_as_float(st[4]);
+            float d2 = fmaf(-2.f, kkb, n2) + ksq;
+            if (d2 < 0.015625f * (n2 + ksq)) {
+              // cancellation regime: recompute |k - kbar|^2 from the key row
+              const uint4* row = reinterpret_cast<const uint4*>(a.K) + ((size_t)u * a.N + i) * 16;
+              float dp[4] = {0.f, 0.f, 0.f, 0.f};
+              for (int c = 0; c < 16; ++c) {
+                const uint4 kv = __ldg(row + c);
+                const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+                for (int t2 = 0; t2 < 4; ++t2) {
+                  const float dl = __uint_as_float(w4[t2] << 16) - kbv[c * 8 + 2 * t2];
+                  const float dh = __uint_as_float(w4[t2] & 0xffff0000u) - kbv[c * 8 + 2 * t2 + 1];
+                  dp[t2] = fmaf(dl, dl, dp[t2]);
+                  dp[t2] = fmaf(dh, dh, dp[t2]);
+                }
+              }
+              d2 = (dp[0] + dp[1]) + (dp[2] + dp[3]);
+            }
+            const float dEv = sqrtf(fmaxf(d2, 0.f));
             const float cs = kmu * (1.f / fmaxf(sqrtf(n2), 1e-12f));
             s_all += dEv;
             if (i < a.Tv) {
@@ -643,30 +748,41 @@ __global__ void __launch_bounds__(kThreads, 1) tc_evict_kernel(const __grid_cons
             }
           }
           ++tcount;
-          if (++stage == kStages) {
-            stage = 0;
-            sphase ^= 1u;
-          }
         }
         if (!ok) break;
-        s_all = group_reduce<Op::Sum, EpiSync>(s_all, s.shf, tid, kEpi);
-        mn = group_reduce<Op::Min, EpiSync>(mn, s.shf, tid, kEpi);
-        mx = group_reduce<Op::Max, EpiSync>(mx, s.shf, tid, kEpi);
-        s_de = group_reduce<Op::Sum, EpiSync>(s_de, s.shf, tid, kEpi);
-        s_c = group_reduce<Op::Sum, EpiSync>(s_c, s.shf, tid, kEpi);
-        s_raw = group_reduce<Op::Sum, EpiSync>(s_raw, s.shf, tid, kEpi);
-        if (tid == 0) {
+        // the chunk's six partials in one pass: warp butterflies, then the
+        // first warp combines the eight warps in a fixed order
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          s_all += __shfl_xor_sync(0xffffffffu, s_all, o);
+          mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+          s_de += __shfl_xor_sync(0xffffffffu, s_de, o);
+          s_c += __shfl_xor_sync(0xffffffffu, s_c, o);
+          s_raw += __shfl_xor_sync(0xffffffffu, s_raw, o);
+        }
+        if (lane == 0) {
+          s.red6[e][0] = s_all;
+          s.red6[e][1] = mn;
+          s.red6[e][2] = mx;
+          s.red6[e][3] = s_de;
+          s.red6[e][4] = s_c;
+          s.red6[e][5] = s_raw;
+        }
+        named_bar_sync(kEpiBar, kEpi);
+        if (tid < 6) {
+          float acc = s.red6[0][tid];
+#pragma unroll
+          for (int w8 = 1; w8 < 8; ++w8) {
+            const float x = s.red6[w8][tid];
+            acc = tid == 1 ? fminf(acc, x) : tid == 2 ? fmaxf(acc, x) : acc + x;
+          }
           float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kP2Stride;
-          p[P2_SUM_DE_ALL] = s_all;
-          p[P2_MIN_DE] = mn;
-          p[P2_MAX_DE] = mx;
-          p[P2_SUM_DE] = s_de;
-          p[P2_SUM_COS] = s_c;
-          p[P2_SUM_RAW] = s_raw;
+          p[tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
         }
       }
-      named_bar_sync(kEpiBar, kEpi);
-      if (tid == 0) mbar_arrive(&s.item_empty[slot]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
     }
   }
 
@@ -682,15 +798,15 @@ int g_num_sms[64] = {0};
 bool g_attr_set[64][4] = {};
 
 template <int RH>
-cudaError_t launch_rh(const CUtensorMap& tm, const TcArgs& a, int dev, cudaStream_t st) {
-  const size_t smem = sizeof(Smem) + 1024;
+cudaError_t launch_rh(const CUtensorMap& tm, const CUtensorMap& tq, const TcArgs& a, int dev, cudaStream_t st) {
+  const size_t smem = sizeof(Smem<RH>) + 1024;
   const int rh_i = RH == 8 ? 0 : RH == 16 ? 1 : RH == 32 ? 2 : 3;
   if (!g_attr_set[dev][rh_i]) {
     cudaError_t e = cudaFuncSetAttribute(tc_evict_kernel<RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     g_attr_set[dev][rh_i] = true;
   }
-  tc_evict_kernel<RH><<<g_num_sms[dev], kThreads, smem, st>>>(tm, a);
+  tc_evict_kernel<RH><<<g_num_sms[dev], kThreads, smem, st>>>(tm, tq, a);
   return cudaGetLastError();
 }
 
@@ -713,12 +829,12 @@ EncodeTiledFn encode_fn() {
 
 }  // namespace
 
-size_t tc_smem_bytes() { return sizeof(Smem) + 1024; }
+size_t tc_smem_bytes() { return sizeof(Smem<32>) + 1024; }
 
 int tc_rows_half(int R) {
   const int r4 = (R + 3) & ~3;
   int np = 16;
-  while (np < r4 + 4) np <<= 1;
+  while (np < r4 + 5) np <<= 1;
   return np > kNPMax ? 0 : np / 2;
 }
 
@@ -742,11 +858,21 @@ cudaError_t launch_tc(const void* K, const TcArgs& args, cudaStream_t st) {
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
+  // window queries as a 2-D [L * h_q * W rows, 128] bf16 tensor, boxes of
+  // [NP rows x 64 columns] with the same 128-byte swizzle as the key tiles
+  CUtensorMap tq;
+  const cuuint64_t qdims[2] = {(cuuint64_t)kD, (cuuint64_t)args.q_rows};
+  const cuuint64_t qstrides[1] = {(cuuint64_t)kD * 2};
+  const cuuint32_t qbox[2] = {64, (cuuint32_t)args.NP};
+  if (enc(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(args.Q), qdims, qstrides, qbox, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
   switch (args.NP / 2) {
-    case 8: return launch_rh<8>(tm, args, dev, st);
-    case 16: return launch_rh<16>(tm, args, dev, st);
-    case 32: return launch_rh<32>(tm, args, dev, st);
-    case 64: return launch_rh<64>(tm, args, dev, st);
+    case 8: return launch_rh<8>(tm, tq, args, dev, st);
+    case 16: return launch_rh<16>(tm, tq, args, dev, st);
+    case 32: return launch_rh<32>(tm, tq, args, dev, st);
+    case 64: return launch_rh<64>(tm, tq, args, dev, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -5,18 +5,22 @@
 
 namespace ecokv {
 
-constexpr int kTcTilesPerChunk = 8;            // 1024 keys per pass item
-constexpr int kTcChunk = 128 * kTcTilesPerChunk;
+constexpr int kTcTilesPerChunk = 8;            // default tiles of 128 keys per pass item
+constexpr int kTcMinTiles = 2;                 // smallest item the workspace is sized for
+constexpr int kTcChunk = 128 * kTcMinTiles;
 
 struct TcArgs {
   int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
+  int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
   int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1
-  int step_items, total_tickets;
+  int total_tickets;                // (U + lag_p2) * 2 * nchunks
   int p1_stride, ustat_stride;
   float scale_log2;
   long long timeout_cycles;
   const void* Q;
+  const void* K;                    // keys, for the direct distance fallback
+  float* norm2;                     // [U][N] squared key norms written by pass 1
   float* p1part;
   float* ustat;
   float* p2part;
