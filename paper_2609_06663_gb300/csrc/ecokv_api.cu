@@ -164,7 +164,7 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.q_rows = p.n_layers * p.h_q * p.window;
   a.tiles_per_chunk = tiles;
   a.nchunks = L.nchunks;
-  a.lag_p2 = env_int("ECOKV_LAG_P2", 8, 1, 64);
+  a.lag_p2 = env_int("ECOKV_LAG_P2", 10, 1, 64);
   a.total_tickets = (L.U + a.lag_p2) * 2 * a.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;

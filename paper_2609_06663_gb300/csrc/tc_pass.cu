@@ -30,8 +30,9 @@
 // tiles into a 4-stage ring; warp 1 issues the tcgen05 MMAs into up to four
 // TMEM accumulators (plus two for the sums); warps 2-3 (key warps) compute
 // the key norms and the sum weights of each pass-1 tile as soon as it lands,
-// so that a ring stage is freed without waiting for the softmax; warps 4-11
-// are the epilogue (one key per TMEM lane, window rows split in two halves).  Every mbarrier wait and spin
+// so that a ring stage is freed without waiting for the softmax, and store
+// the norms for pass 2; warps 4-11 are the epilogue (one key per TMEM lane,
+// window rows split in two halves).  Every mbarrier wait and spin
 // is bounded: on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
 // gpu-wide abort flag, drains its own copies and MMAs, frees TMEM and exits.
 
@@ -87,6 +88,7 @@ struct __align__(1024) Smem {
   uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
   uint64_t tmem_full[4], tmem_empty[4];
   uint64_t sigma_full[2], sigma_empty[2], drain;
+  uint64_t kpub[kIQ];  // key warps have published this item's key norms (gpu scope)
   uint32_t tmem_base;
   int flag_last;
 };
@@ -294,6 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&s.sigma_full[i], 1);
       mbar_init(&s.sigma_empty[i], 4);
     }
+    for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], 2);  // 2 key warps
     mbar_init(&s.drain, 1);
     fence_mbar_init();
   }
@@ -324,6 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int stage = 0;
     uint32_t sphase = 0;
     uint32_t used_bits = 0u, par_bits = 0u;  // per stage: loaded at least once / parity of loads
+    const uint64_t pol_keep = l2_policy_evict_last(), pol_drop = l2_policy_evict_first();
     for (int seq = 0; ok;) {
       int ticket = 0;
       if (lane == 0) ticket = (int)atomicAdd(a.sync, 1u);
@@ -377,8 +381,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (ok) {
             mbar_expect_tx(&s.full[stage], kTileBytes);
             const int y = i0 + t * kTile;
-            tma_load_3d(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u);
-            tma_load_3d(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u);
+            // pass 1 keeps its keys in L2 for pass 2; pass 2 reads them for the last time
+            const uint64_t pol = it.type == kP1 ? pol_keep : pol_drop;
+            tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u, pol);
+            tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u, pol);
             used_bits |= 1u << stage;
             par_bits ^= 1u << stage;
           }
@@ -482,12 +488,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = 0; t < ntiles && ok; ++t) {
         if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
         if (type == kP1) {
-          // squared norms, the sum weights w = 1/||k|| (three bf16 terms) and
-          // the norms for pass 2
+          // squared norms (packed fp32 pairs), the sum weights w = 1/||k|| in
+          // three bf16 terms, and the norms for pass 2
 #pragma unroll
           for (int q2 = 0; q2 < 2; ++q2) {
             const int kk = tk + 64 * q2;
-            float n2p[4] = {0.f, 0.f, 0.f, 0.f};
+            uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
             for (int hb = 0; hb < 2; ++hb) {
               const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
@@ -497,13 +503,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
                 for (int t2 = 0; t2 < 4; ++t2) {
-                  const float lo = __uint_as_float(w4[t2] << 16), hi = __uint_as_float(w4[t2] & 0xffff0000u);
-                  n2p[t2] = fmaf(lo, lo, n2p[t2]);
-                  n2p[t2] = fmaf(hi, hi, n2p[t2]);
+                  const uint64_t x = pack_f32x2(__uint_as_float(w4[t2] << 16), __uint_as_float(w4[t2] & 0xffff0000u));
+                  acc[t2] = ffma2(x, x, acc[t2]);
                 }
               }
             }
-            const float n2 = (n2p[0] + n2p[1]) + (n2p[2] + n2p[3]);
+            const float n2 = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
+                             ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
             const int i = i0 + t * kTile + kk;
             const bool valid = i < a.N;
             if (valid) a.norm2[(size_t)u * a.N + i] = n2;
@@ -518,7 +524,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
             *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;
           }
-          __threadfence();  // key norms visible before the unit's pass-1 arrival count
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.wready[stage]);
@@ -531,8 +536,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) break;
+      // publish this item's key norms at gpu scope (the fence is cumulative
+      // over the warp's stores ordered before it by __syncwarp)
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
+      if (lane == 0) {
+        if (type == kP1) __threadfence();
+        mbar_arrive(&s.kpub[slot]);
+        mbar_arrive(&s.item_empty[slot]);
+      }
     }
   } else {
     // ------------------------------------------------ epilogue (warps 4..11)
@@ -577,26 +588,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           m[c] = -INFINITY;
           z[c] = 0.f;
         }
+        const uint32_t bmask = (1u << nbuf_log) - 1u;
         for (int t = 0; t < ntiles && ok; ++t) {
           const int it0 = i0 + t * kTile;
           const int i = it0 + kk;
           const bool valid = i < a.N;
-          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
+          const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 12u))) break;
           tc_fence_after();
-          uint32_t r[RH];
-          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), r);
+          uint32_t rc[RH];
+          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), rc);
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
+          ++tcount;
           // online softmax partials, branch-free: re-base the running sum only
           // when a logit exceeds the running reference by more than 2^20
           if (it0 + kTile - 1 <= a.N - a.W) {
             // every key of the tile is visible to every window row
 #pragma unroll
             for (int c = 0; c < RH; ++c) {
-              const float x = __uint_as_float(r[c]) * a.scale_log2;
+              const float x = __uint_as_float(rc[c]) * a.scale_log2;
               const float dlt = (h * RH + c < a.R) ? x - m[c] : -INFINITY;
               const bool up = dlt > 20.f;
               const float ee = ex2(up ? -dlt : dlt);
@@ -612,7 +625,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < RH; ++c) {
               const bool vis = (h * RH + c < a.R) && valid && j >= vis_from;
               if (++j == a.W) j = 0;
-              const float x = __uint_as_float(r[c]) * a.scale_log2;
+              const float x = __uint_as_float(rc[c]) * a.scale_log2;
               const float dlt = vis ? x - m[c] : -INFINITY;
               const bool up = dlt > 20.f;
               const float ee = ex2(up ? -dlt : dlt);
@@ -620,7 +633,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               m[c] = up ? x : m[c];
             }
           }
-          ++tcount;
         }
         if (!ok) break;
         // item end: per-row (max, sum) over the 32 keys of the warp, step-major
@@ -678,9 +690,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           part[2 * a.R + kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
         }
         ++sigcount;
-        __threadfence();  // this thread's partials before the arrival count
+        if (tid < a.R || h == 0) __threadfence();  // this thread's partials before the arrival count
         named_bar_sync(kEpiBar, kEpi);
-        if (tid == 0) pending_old = atom_add_acq_rel(a.sync + 4 + u, 1u);  // resolved at the next loop top
+        if (tid == 0) {
+          // the key norms of this item are published too
+          ok = wait_bar(&s.kpub[slot], qphase, a, 19u);
+          if (ok) pending_old = atom_add_acq_rel(a.sync + 4 + u, 1u);  // resolved at the next loop top
+        }
         pending_u = u;
       } else {  // kP2
         if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 18u))) break;  // statistics copy landed
@@ -688,32 +704,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float* kbv = d.ust + ustat_kbar();
         const float ksq = d.ust[ustat_ksq()];
         float s_all = 0.f, mn = INFINITY, mx = -INFINITY, s_de = 0.f, s_c = 0.f, s_raw = 0.f;
+        const uint32_t bmask = (1u << nbuf_log) - 1u;
         for (int t = 0; t < ntiles && ok; ++t) {
           const int i = i0 + t * kTile + kk;
           const bool valid = i < a.N;
-          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
+          const float n2 = (h == 0 && valid) ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;  // in flight early
+          const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 14u))) break;
           tc_fence_after();
-          uint32_t r[RH], st[8];
-          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), r);
-          if (h == 0) tmem_ld_x8(tl + b * (uint32_t)a.NP + (uint32_t)a.R4, st);
-          const float n2 = (h == 0 && valid) ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;
+          uint32_t rc[RH], stc[8];
+          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), rc);
+          if (h == 0) tmem_ld_x8(tl + b * (uint32_t)a.NP + (uint32_t)a.R4, stc);
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
+          const uint32_t par = tcount & 1u;
+          ++tcount;
           float vp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < RH; ++c) {
             const int rowi = h * RH + c;
-            if (rowi < a.R) vp[c & 3] += ex2(fmaf(__uint_as_float(r[c]), a.scale_log2, -lse[rowi]));
+            if (rowi < a.R) vp[c & 3] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -lse[rowi]));
           }
-          s.xch[tcount & 1u][h][kk] = (vp[0] + vp[1]) + (vp[2] + vp[3]);
+          s.xch[par][h][kk] = (vp[0] + vp[1]) + (vp[2] + vp[3]);
           named_bar_sync(kEpiBar, kEpi);
           if (h == 0 && valid) {
-            const float v = s.xch[tcount & 1u][0][kk] + s.xch[tcount & 1u][1][kk];
-            const float kkb = (__uint_as_float(st[0]) + __uint_as_float(st[1])) + __uint_as_float(st[2]);
-            const float kmu = __uint_as_float(st[3]) + __uint_as_float(st[4]);
+            const float v = s.xch[par][0][kk] + s.xch[par][1][kk];
+            const float kkb = (__uint_as_float(stc[0]) + __uint_as_float(stc[1])) + __uint_as_float(stc[2]);
+            const float kmu = __uint_as_float(stc[3]) + __uint_as_float(stc[4]);
             float d2 = fmaf(-2.f, kkb, n2) + ksq;
             if (d2 < 0.015625f * (n2 + ksq)) {
               // cancellation regime: recompute |k - kbar|^2 from the key row
@@ -747,7 +766,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               a.cosv[o] = cs;
             }
           }
-          ++tcount;
         }
         if (!ok) break;
         // the chunk's six partials in one pass: warp butterflies, then the
