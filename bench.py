@@ -76,11 +76,11 @@ def byte_model(w) -> dict:
 
 def launches_per_call(w) -> int:
     """Kernels one ecokv_evict call launches: the persistent tensor-core
-    streaming kernel (bf16, n >= 128, g*W <= 124) or the two CUDA-core passes,
-    then the finalize/select/compact kernel."""
+    streaming kernel (bf16, n >= 128, g*W <= 120) or the two CUDA-core passes,
+    then the finalize/select kernel and the compaction kernel."""
     r = w.group * w.window
-    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 4 <= 128
-    return 2 if tc else 3
+    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 5 <= 128
+    return 3 if tc else 4
 
 
 def measured_peaks() -> tuple[float, str]:

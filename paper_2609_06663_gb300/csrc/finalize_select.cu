@@ -8,10 +8,10 @@ namespace {
 
 constexpr int kFinThreads = 1024;
 
-// Scores of unit blockIdx.x; with kSelect the top-k, with kCompact the gather
-// of the retained rows.  kSmem keeps the unit's scores in shared memory.
-template <typename T, bool kSmem, bool kSelect, bool kCompact>
-__global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalArgs f, CompactArgs c) {
+// Scores of unit blockIdx.x and, with kSelect, its top-k.  kSmem keeps the
+// unit's scores in shared memory.
+template <bool kSmem, bool kSelect>
+__global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalArgs f) {
   extern __shared__ float sS[];
   __shared__ float shf[64];
   __shared__ unsigned hist[256];
@@ -20,10 +20,6 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(FinalArgs f, Comp
   float* S = kSmem ? sS : (f.S ? f.S : f.S_scratch) + (size_t)u * f.Tv;
   finalize_unit<BlockSync>(f, u, S, shf, threadIdx.x, blockDim.x);
   if (kSelect) select_unit<BlockSync>(f, u, S, hist, shi, threadIdx.x, blockDim.x);
-  if (kCompact) {
-    __syncthreads();
-    gather_rows<T>(c, u, 0, f.n_keep, threadIdx.x, blockDim.x);
-  }
 }
 
 __global__ void __launch_bounds__(kFinThreads) select_kernel(FinalArgs f) {
@@ -40,30 +36,28 @@ __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a) {
   gather_rows<T>(a, blockIdx.y, r0, r0 + rows, threadIdx.x, blockDim.x);
 }
 
-template <typename T>
-cudaError_t launch_fc(const FinalArgs& f, const CompactArgs& c, int U, cudaStream_t s) {
-  if (f.Tv > 0 && f.Tv <= kSmemScores) {
-    const size_t smem = (size_t)f.Tv * sizeof(float);
-    cudaError_t e =
-        cudaFuncSetAttribute(finalize_kernel<T, true, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-    if (e != cudaSuccess) return e;
-    finalize_kernel<T, true, true, true><<<U, kFinThreads, smem, s>>>(f, c);
-  } else {
-    finalize_kernel<T, false, true, true><<<U, kFinThreads, 0, s>>>(f, c);
-  }
-  return cudaGetLastError();
-}
-
 }  // namespace
 
+// Scores (and with a compaction target, the top-k and the gather of the kept
+// rows, the gather as its own many-CTA launch so that every SM streams rows).
 cudaError_t launch_finalize(const FinalArgs& f, const CompactArgs* c, ecokv_dtype dt, int U, bool do_select,
                             cudaStream_t s) {
   if (!do_select || c == nullptr) {
-    finalize_kernel<float, false, false, false><<<U, kFinThreads, 0, s>>>(f, CompactArgs{});
+    finalize_kernel<false, false><<<U, kFinThreads, 0, s>>>(f);
     return cudaGetLastError();
   }
-  return dt == ECOKV_F32 ? launch_fc<float>(f, *c, U, s) : launch_fc<__nv_bfloat16>(f, *c, U, s);
+  if (f.Tv > 0 && f.Tv <= kSmemScores) {
+    const size_t smem = (size_t)f.Tv * sizeof(float);
+    cudaError_t e =
+        cudaFuncSetAttribute(finalize_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    finalize_kernel<true, true><<<U, kFinThreads, smem, s>>>(f);
+  } else {
+    finalize_kernel<false, true><<<U, kFinThreads, 0, s>>>(f);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_compact(*c, dt, U, s);
 }
 
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s) {

@@ -138,13 +138,27 @@ __device__ void finalize_unit(const FinalArgs& a, int u, float* Sbuf, float* shf
   if (Tv == 0) return;
   const float denE = __fadd_rn(__fsub_rn(mxE, mnE), a.eps);
 
-  // sweep 1: extrema of S_div, pooled importance into Sbuf
+  // sweep 1: extrema of S_div, pooled importance into Sbuf (four candidates
+  // per thread in flight)
   float mnD = INFINITY, mxD = -INFINITY;
-  for (int i = tid; i < Tv; i += nt) {
-    const float sd = sdiv_of(__ldg(dE + i), __ldg(cv + i), mnE, denE, a.alpha, mix);
-    mnD = fminf(mnD, sd);
-    mxD = fmaxf(mxD, sd);
-    Sbuf[i] = pooled(raw, i, Tv, a.pool);
+  for (int i0 = tid; i0 < Tv; i0 += 4 * nt) {
+    float e4[4], c4[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * nt;
+      e4[q] = i < Tv ? __ldg(dE + i) : 0.f;
+      c4[q] = i < Tv ? __ldg(cv + i) : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * nt;
+      if (i < Tv) {
+        const float sd = sdiv_of(e4[q], c4[q], mnE, denE, a.alpha, mix);
+        mnD = fminf(mnD, sd);
+        mxD = fmaxf(mxD, sd);
+        Sbuf[i] = pooled(raw, i, Tv, a.pool);
+      }
+    }
   }
   mnD = group_reduce<Op::Min, Sync>(mnD, shf, tid, nt);
   mxD = group_reduce<Op::Max, Sync>(mxD, shf, tid, nt);
@@ -172,20 +186,32 @@ __device__ void finalize_unit(const FinalArgs& a, int u, float* Sbuf, float* shf
   const float one_m_lam = __fsub_rn(1.f, lamf);
 
   // sweep 2: final score (Eq. 7)
-  for (int i = tid; i < Tv; i += nt) {
-    const float e = __ldg(dE + i), c = __ldg(cv + i);
-    const float sd = sdiv_of(e, c, mnE, denE, a.alpha, mix);
-    const float sbar = __fdiv_rn(__fsub_rn(sd, mnD), denD);
-    const float sp = Sbuf[i];
-    const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
-    Sbuf[i] = S;
-    if (Sg) Sg[i] = S;
-    if (dbg) {
-      dbg[i] = __ldg(raw + i);
-      dbg[Tv + i] = sp;
-      dbg[2 * Tv + i] = e;
-      dbg[3 * Tv + i] = c;
-      dbg[4 * Tv + i] = sd;
+  for (int i0 = tid; i0 < Tv; i0 += 4 * nt) {
+    float e4[4], c4[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * nt;
+      e4[q] = i < Tv ? __ldg(dE + i) : 0.f;
+      c4[q] = i < Tv ? __ldg(cv + i) : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * nt;
+      if (i < Tv) {
+        const float sd = sdiv_of(e4[q], c4[q], mnE, denE, a.alpha, mix);
+        const float sbar = __fdiv_rn(__fsub_rn(sd, mnD), denD);
+        const float sp = Sbuf[i];
+        const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
+        Sbuf[i] = S;
+        if (Sg) Sg[i] = S;
+        if (dbg) {
+          dbg[i] = __ldg(raw + i);
+          dbg[Tv + i] = sp;
+          dbg[2 * Tv + i] = e4[q];
+          dbg[3 * Tv + i] = c4[q];
+          dbg[4 * Tv + i] = sd;
+        }
+      }
     }
   }
   Sync::sync();
