@@ -132,6 +132,33 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
                          const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
                          float* lambda, void* ws, size_t ws_bytes, void* stream);
 
+/* ecokv_evict without a caller workspace and without any allocation.  The
+ * paper has no counterpart: this is a deployment variant of the same pass for
+ * callers that may not allocate device memory where they evict (a runtime
+ * that gave all free HBM to its KV-cache pool, or C code with no allocator).
+ *
+ * The workspace is a fixed scratch area of ECOKV_NOALLOC_SCRATCH_BYTES
+ * compiled into the library, one copy per device context, loaded with the
+ * library's module on first use.  Nothing is allocated by the call: no
+ * cudaMalloc, no allocating library routine.
+ *   Arguments as for ecokv_evict, minus ws / ws_bytes, plus
+ *   dev_status : optional (NULL to skip) device pointer, 4-byte aligned; in
+ *                stream order after the pass it receives the call's device-side
+ *                status (0, ECOKV_ERR_TIMEOUT or ECOKV_ERR_DEVICE_INDEX).
+ * Errors: everything ecokv_evict returns; ECOKV_ERR_WORKSPACE when the
+ * workspace *p needs (ecokv_workspace_size) exceeds
+ * ECOKV_NOALLOC_SCRATCH_BYTES, checked before anything is launched;
+ * ECOKV_ERR_CUDA when the scratch's address cannot be obtained.
+ * Set-up: the first call on a device looks the scratch's address up (with
+ * that device current); make that first call before any stream capture.
+ * Concurrency: all calls on one device share the scratch.  Calls whose
+ * executions may overlap (unordered streams, several host threads) race on
+ * it; issue them in one stream order. */
+#define ECOKV_NOALLOC_SCRATCH_BYTES (16u << 20)
+ecokv_status ecokv_evict_noalloc(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                                 const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
+                                 float* lambda, uint32_t* dev_status, void* stream);
+
 /* Synchronise `stream`, then read and clear the workspace's device status
  * word.  Returns ECOKV_OK, ECOKV_ERR_DEVICE_INDEX, ECOKV_ERR_TIMEOUT, or
  * ECOKV_ERR_CUDA if the synchronisation itself failed. */

@@ -16,12 +16,16 @@ ECOKV_F32, ECOKV_BF16 = 0, 1
 ECOKV_FLAG_SC_MIXKV_SIGN = 0x1
 ECOKV_FLAG_LAMBDA_OVERRIDE = 0x2
 ECOKV_FLAG_FORCE_SIMT = 0x100
+ECOKV_NOALLOC_SCRATCH_BYTES = 16 << 20   # fixed scratch of ecokv_evict_noalloc, per device
+ECOKV_OK, ECOKV_ERR_INVALID_ARG, ECOKV_ERR_UNSUPPORTED, ECOKV_ERR_WORKSPACE = 0, 1, 2, 3
+ECOKV_ERR_CUDA, ECOKV_ERR_TIMEOUT, ECOKV_ERR_DEVICE_INDEX = 4, 5, 6
 
 STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED", 3: "ECOKV_ERR_WORKSPACE",
           4: "ECOKV_ERR_CUDA", 5: "ECOKV_ERR_TIMEOUT", 6: "ECOKV_ERR_DEVICE_INDEX"}
 
 EXPORTS = ("ecokv_params_default", "ecokv_check_params", "ecokv_workspace_size", "ecokv_score",
-           "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string")
+           "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string",
+           "ecokv_evict_noalloc")
 
 
 class EcokvError(RuntimeError):
@@ -68,6 +72,8 @@ def lib() -> ctypes.CDLL:
         L.ecokv_compact.restype = ctypes.c_int
         L.ecokv_evict.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
         L.ecokv_evict.restype = ctypes.c_int
+        L.ecokv_evict_noalloc.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
+        L.ecokv_evict_noalloc.restype = ctypes.c_int
         L.ecokv_device_status.argtypes = [_vp, _vp]
         L.ecokv_device_status.restype = ctypes.c_int
         L.ecokv_status_string.argtypes = [ctypes.c_int]
@@ -133,6 +139,12 @@ def ecokv_compact(p, dtype, K, V, idx, K_out, V_out, ws=None, ws_bytes=0, stream
 def ecokv_evict(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, ws, ws_bytes, stream=None) -> int:
     return lib().ecokv_evict(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx), _ptr(K_out),
                              _ptr(V_out), _ptr(S), _ptr(lam), _ptr(ws), ws_bytes, _stream(stream))
+
+
+def ecokv_evict_noalloc(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, dev_status, stream=None) -> int:
+    return lib().ecokv_evict_noalloc(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx),
+                                     _ptr(K_out), _ptr(V_out), _ptr(S), _ptr(lam), _ptr(dev_status),
+                                     _stream(stream))
 
 
 def ecokv_device_status(ws, stream=None) -> int:
@@ -210,3 +222,20 @@ def evict(p, K, V, Qwin, ws=None, want_scores=False, stream=None):
     _check(ecokv_evict(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, ws, ws.numel(), stream),
            "ecokv_evict")
     return idx, Ko, Vo, S, lam
+
+
+def evict_noalloc(p, K, V, Qwin, want_scores=False, stream=None):
+    """Run ecokv_evict_noalloc (library-held scratch, no workspace argument);
+    returns (idx, K_out, V_out, S or None, lambda, device status code)."""
+    import torch
+    n_keep = min(p.budget, p.n)
+    idx = torch.empty(p.n_layers, p.h_kv, n_keep, dtype=torch.int32, device=K.device)
+    Ko = torch.empty(p.n_layers, p.h_kv, n_keep, p.d, dtype=K.dtype, device=K.device)
+    Vo = torch.empty_like(Ko)
+    S = torch.empty(p.n_layers, p.h_kv, p.n - p.window, dtype=torch.float32, device=K.device) \
+        if want_scores else None
+    lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32, device=K.device)
+    code = torch.full((1,), -1, dtype=torch.int32, device=K.device)
+    _check(ecokv_evict_noalloc(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, code, stream),
+           "ecokv_evict_noalloc")
+    return idx, Ko, Vo, S, lam, int(code.item())

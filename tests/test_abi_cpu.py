@@ -101,3 +101,9 @@ def test_no_cpu_fallback_when_library_missing(monkeypatch, tmp_path):
     monkeypatch.setattr(E, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         E.lib()
+
+
+def test_binding_constants_match_header():
+    txt = open(os.path.join(ROOT, "include", "ecokv.h")).read()
+    m = re.search(r"#define ECOKV_NOALLOC_SCRATCH_BYTES \((\d+)u << (\d+)\)", txt)
+    assert m and int(m.group(1)) << int(m.group(2)) == E.ECOKV_NOALLOC_SCRATCH_BYTES
