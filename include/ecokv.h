@@ -164,6 +164,16 @@ ecokv_status ecokv_evict_noalloc(const ecokv_params* p, ecokv_dtype dtype, const
  * ECOKV_ERR_CUDA if the synchronisation itself failed. */
 ecokv_status ecokv_device_status(void* ws, void* stream);
 
+/* Timing hook for benchmarks and profiling (no counterpart in the paper).
+ * events: NULL to switch the hook off, else 4 cudaEvent_t handles created and
+ * owned by the caller (n must be 4).  While set, every ecokv_score /
+ * ecokv_evict call made from this host thread records, on its stream,
+ * events[0] before the streaming kernel(s), events[1] after them, events[2]
+ * after the finalize / select kernel and (ecokv_evict only) events[3] after
+ * the compaction kernel, so that cudaEventElapsedTime gives each stage's
+ * device time.  Returns ECOKV_ERR_INVALID_ARG if events != NULL and n != 4. */
+ecokv_status ecokv_set_stage_events(void* const* events, int n);
+
 /* Static text for a status code. */
 const char* ecokv_status_string(ecokv_status s);
 

@@ -68,6 +68,14 @@ static bool use_tensor_path(const ecokv_params& p, ecokv_dtype dt) {
 
 static int env_int(const char* name, int dflt, int lo, int hi);
 
+// Stage events of this host thread (ecokv_set_stage_events), recorded on the
+// call's stream between its launches when set.
+thread_local cudaEvent_t g_stage_ev[4] = {nullptr, nullptr, nullptr, nullptr};
+
+static void stage_event(int i, cudaStream_t s) {
+  if (g_stage_ev[i] != nullptr) cudaEventRecord(g_stage_ev[i], s);
+}
+
 // Keys per tensor-core pass item (128 * tiles; ECOKV_TC_TILES overrides the
 // default of 8 tiles for tuning).
 static int tc_chunk_keys() { return 128 * env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64); }
@@ -255,9 +263,12 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   f.S = S;
   f.lambda = lambda;
   f.dbg = dbg;
+  stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
-  if (launch_finalize(f, nullptr, dtype, L.U, false, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(1, s);
+  if (launch_finalize(f, L.U, false, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(2, s);
   return ECOKV_OK;
 }
 
@@ -315,9 +326,14 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   f.lambda = lambda;
   f.idx = idx;
   const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, reinterpret_cast<unsigned*>(w + L.status));
+  stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
-  if (launch_finalize(f, &c, dtype, L.U, true, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(1, s);
+  if (launch_finalize(f, L.U, true, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(2, s);
+  if (launch_compact(c, dtype, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(3, s);
   return ECOKV_OK;
 }
 
@@ -332,6 +348,16 @@ ecokv_status ecokv_device_status(void* ws, void* stream) {
     if (cudaMemcpy(ws, &z, sizeof(z), cudaMemcpyHostToDevice) != cudaSuccess) return ECOKV_ERR_CUDA;
   }
   return static_cast<ecokv_status>(h.code);
+}
+
+ecokv_status ecokv_set_stage_events(void* const* events, int n) {
+  if (events == nullptr) {
+    for (int i = 0; i < 4; ++i) g_stage_ev[i] = nullptr;
+    return ECOKV_OK;
+  }
+  if (n != 4) return ECOKV_ERR_INVALID_ARG;
+  for (int i = 0; i < 4; ++i) g_stage_ev[i] = static_cast<cudaEvent_t>(events[i]);
+  return ECOKV_OK;
 }
 
 const char* ecokv_status_string(ecokv_status s) {

@@ -105,8 +105,7 @@ struct CompactArgs {
 // launchers (return cudaGetLastError() after the launch)
 cudaError_t launch_score_simt(const ScoreArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
 // finalize (scores), then optionally select and gather, one CTA per unit
-cudaError_t launch_finalize(const FinalArgs& f, const CompactArgs* c, ecokv_dtype dt, int U, bool do_select,
-                            cudaStream_t s);
+cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStream_t s);
 // select only, on caller scores f.S
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s);
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s);

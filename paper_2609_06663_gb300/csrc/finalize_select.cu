@@ -1,5 +1,5 @@
-// Finalisation, selection and compaction kernels (one CTA per unit); the
-// device code lives in finalize_select.cuh.
+// Finalisation and selection kernels (one CTA per unit) and the compaction
+// kernel (32 kept rows per CTA); the device code lives in finalize_select.cuh.
 
 #include "finalize_select.cuh"
 
@@ -38,11 +38,9 @@ __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a) {
 
 }  // namespace
 
-// Scores (and with a compaction target, the top-k and the gather of the kept
-// rows, the gather as its own many-CTA launch so that every SM streams rows).
-cudaError_t launch_finalize(const FinalArgs& f, const CompactArgs* c, ecokv_dtype dt, int U, bool do_select,
-                            cudaStream_t s) {
-  if (!do_select || c == nullptr) {
+// Scores of every unit and, with do_select, their top-k.
+cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStream_t s) {
+  if (!do_select) {
     finalize_kernel<false, false><<<U, kFinThreads, 0, s>>>(f);
     return cudaGetLastError();
   }
@@ -55,9 +53,7 @@ cudaError_t launch_finalize(const FinalArgs& f, const CompactArgs* c, ecokv_dtyp
   } else {
     finalize_kernel<false, true><<<U, kFinThreads, 0, s>>>(f);
   }
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  return launch_compact(*c, dt, U, s);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s) {

@@ -25,7 +25,7 @@ STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED",
 
 EXPORTS = ("ecokv_params_default", "ecokv_check_params", "ecokv_workspace_size", "ecokv_score",
            "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string",
-           "ecokv_evict_noalloc")
+           "ecokv_evict_noalloc", "ecokv_set_stage_events")
 
 
 class EcokvError(RuntimeError):
@@ -74,6 +74,8 @@ def lib() -> ctypes.CDLL:
         L.ecokv_evict.restype = ctypes.c_int
         L.ecokv_evict_noalloc.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
         L.ecokv_evict_noalloc.restype = ctypes.c_int
+        L.ecokv_set_stage_events.argtypes = [ctypes.POINTER(_vp), ctypes.c_int]
+        L.ecokv_set_stage_events.restype = ctypes.c_int
         L.ecokv_device_status.argtypes = [_vp, _vp]
         L.ecokv_device_status.restype = ctypes.c_int
         L.ecokv_status_string.argtypes = [ctypes.c_int]
@@ -145,6 +147,15 @@ def ecokv_evict_noalloc(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, dev_sta
     return lib().ecokv_evict_noalloc(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx),
                                      _ptr(K_out), _ptr(V_out), _ptr(S), _ptr(lam), _ptr(dev_status),
                                      _stream(stream))
+
+
+def ecokv_set_stage_events(events) -> int:
+    """events: None (hook off) or 4 torch.cuda.Event objects (or raw handles)."""
+    if events is None:
+        return lib().ecokv_set_stage_events(None, 0)
+    hs = [e.cuda_event if hasattr(e, "cuda_event") else int(e) for e in events]
+    arr = (_vp * len(hs))(*hs)
+    return lib().ecokv_set_stage_events(arr, len(hs))
 
 
 def ecokv_device_status(ws, stream=None) -> int:
@@ -237,5 +248,5 @@ def evict_noalloc(p, K, V, Qwin, want_scores=False, stream=None):
     lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32, device=K.device)
     code = torch.full((1,), -1, dtype=torch.int32, device=K.device)
     _check(ecokv_evict_noalloc(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, code, stream),
-           "ecokv_evict_noalloc")
+           "ecokv_evict_noalloc", "ecokv_set_stage_events")
     return idx, Ko, Vo, S, lam, int(code.item())

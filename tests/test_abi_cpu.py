@@ -107,3 +107,8 @@ def test_binding_constants_match_header():
     txt = open(os.path.join(ROOT, "include", "ecokv.h")).read()
     m = re.search(r"#define ECOKV_NOALLOC_SCRATCH_BYTES \((\d+)u << (\d+)\)", txt)
     assert m and int(m.group(1)) << int(m.group(2)) == E.ECOKV_NOALLOC_SCRATCH_BYTES
+
+
+def test_stage_events_hook_arguments(lib):
+    assert E.ecokv_set_stage_events(None) == 0
+    assert lib.ecokv_set_stage_events((ctypes.c_void_p * 2)(None, None), 2) == 1
