@@ -248,5 +248,5 @@ def evict_noalloc(p, K, V, Qwin, want_scores=False, stream=None):
     lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32, device=K.device)
     code = torch.full((1,), -1, dtype=torch.int32, device=K.device)
     _check(ecokv_evict_noalloc(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, code, stream),
-           "ecokv_evict_noalloc", "ecokv_set_stage_events")
+           "ecokv_evict_noalloc")
     return idx, Ko, Vo, S, lam, int(code.item())
