@@ -59,7 +59,7 @@ __host__ __device__ inline int ustat_kbar() { return 0; }
 __host__ __device__ inline int ustat_mu() { return kD; }
 __host__ __device__ inline int ustat_ksq() { return 2 * kD; }
 __host__ __device__ inline int ustat_musq() { return 2 * kD + 1; }
-__host__ __device__ inline int ustat_lse() { return 2 * kD + 2; }
+__host__ __device__ inline int ustat_lse() { return 2 * kD + 4; }  // 16-byte aligned
 
 struct ScoreArgs {
   const void* K;

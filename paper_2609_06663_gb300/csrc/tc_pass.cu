@@ -61,7 +61,8 @@ constexpr uint32_t kEpiBar = 1;
 
 enum : int { kP1 = 0, kP2 = 1, kExit = 3 };
 
-constexpr int kUstatMax = (2 * kD + 2 + kNPMax + 3) & ~3;  // floats of a unit statistics record
+constexpr int kNB = 4;                // pass-2 norm hand-off slots
+constexpr int kUstatMax = 2 * kD + 4 + kNPMax;  // floats of a unit statistics record (lse padded to NP rows)
 
 struct __align__(16) ItemDesc {
   int type, u, chunk, part, i0, ntiles;
@@ -88,6 +89,8 @@ struct __align__(1024) Smem {
   uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
   uint64_t tmem_full[4], tmem_empty[4];
   uint64_t sigma_full[2], sigma_empty[2], drain;
+  float nbuf[kNB][kTile];                        // pass-2 squared key norms, key warps -> epilogue
+  uint64_t nfull[kNB], nempty[kNB];
   uint64_t kpub[kIQ];  // key warps have published this item's key norms (gpu scope)
   uint32_t tmem_base;
   int flag_last;
@@ -180,7 +183,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // hold kbar split into three bf16 terms (hi, mid, lo), rows R4+3, R4+4 hold
 // mu_hi and mu_lo, all from the unit statistics copy; the window queries in
 // rows 0..R-1 arrive by TMA.  Run by the 32 lanes of warp 0.
-__device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, const float* ust, int lane) {
+__device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, float* ust, int lane) {
+  // rows past the window rows (padding and the statistics rows) get an
+  // infinite log-sum-exp, so that their vote terms are exactly zero
+  for (int r = a.R + lane; r < a.NP; r += 32) ust[ustat_lse() + r] = INFINITY;
   for (int e = lane; e < 5 * 16; e += 32) {
     const int which = e >> 4, j = e & 15;
     const float* src = ust + (which < 3 ? ustat_kbar() : ustat_mu()) + j * 8;
@@ -297,6 +303,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&s.sigma_empty[i], 4);
     }
     for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], 2);  // 2 key warps
+    for (int i = 0; i < kNB; ++i) {
+      mbar_init(&s.nfull[i], 2);   // 2 key warps
+      mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the first row half
+    }
     mbar_init(&s.drain, 1);
     fence_mbar_init();
   }
@@ -477,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ key warps (2..3)
     const int tk = threadIdx.x - 64;  // 0..63: keys tk and tk + 64 of each tile
     int stage = 0;
-    uint32_t sphase = 0;
+    uint32_t sphase = 0, p2count = 0;
     for (int seq = 0; ok; ++seq) {
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
@@ -488,8 +498,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = 0; t < ntiles && ok; ++t) {
         if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
         if (type == kP1) {
-          // squared norms (packed fp32 pairs), the sum weights w = 1/||k|| in
-          // three bf16 terms, and the norms for pass 2
+          // squared norms of this thread's two keys (packed fp32 pairs), kept
+          // for pass 2, and the sum weights w = 1/||k|| in three bf16 terms
+          float n2v[2];
 #pragma unroll
           for (int q2 = 0; q2 < 2; ++q2) {
             const int kk = tk + 64 * q2;
@@ -508,12 +519,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
               }
             }
-            const float n2 = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
-                             ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
+            n2v[q2] = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
+                      ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
+#pragma unroll
+          for (int q2 = 0; q2 < 2; ++q2) {
+            const int kk = tk + 64 * q2;
             const int i = i0 + t * kTile + kk;
             const bool valid = i < a.N;
-            if (valid) a.norm2[(size_t)u * a.N + i] = n2;
-            const float w = valid ? 1.f / fmaxf(sqrtf(n2), 1e-12f) : 0.f;
+            if (valid) a.norm2[(size_t)u * a.N + i] = n2v[q2];
+            const float w = valid ? rsqrtf(fmaxf(n2v[q2], 1e-24f)) : 0.f;
             const __nv_bfloat16 whi = __float2bfloat16_rn(w);
             const float r1 = w - __bfloat162float(whi);
             const __nv_bfloat16 wmid = __float2bfloat16_rn(r1);
@@ -527,17 +544,31 @@ __global__ void __launch_bounds__(kThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.wready[stage]);
+        } else {
+          // pass 2: the keys are only needed by the MMA; the norms pass 1
+          // stored go to the epilogue through shared memory
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.empty[stage]);
+          const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
+          ++p2count;
+          const int ia = i0 + t * kTile + tk, ib = ia + 64;
+          const float na = ia < a.N ? __ldcg(a.norm2 + (size_t)u * a.N + ia) : 0.f;
+          const float nbv = ib < a.N ? __ldcg(a.norm2 + (size_t)u * a.N + ib) : 0.f;
+          if (!(ok = wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u))) break;
+          s.nbuf[nb][tk] = na;
+          s.nbuf[nb][tk + 64] = nbv;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.nfull[nb]);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
         if (++stage == kStages) {
           stage = 0;
           sphase ^= 1u;
         }
       }
       if (!ok) break;
-      // publish this item's key norms at gpu scope (the fence is cumulative
-      // over the warp's stores ordered before it by __syncwarp)
+      // publish this item's key norms at gpu scope before the epilogue counts
+      // the item as arrived (the fence is cumulative over the warp's stores
+      // ordered before it by __syncwarp)
       __syncwarp();
       if (lane == 0) {
         if (type == kP1) __threadfence();
@@ -551,7 +582,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kk = 32 * q + lane;  // key row within a tile = TMEM lane
     const int tid = threadIdx.x - 32 * kEpiWarp0;
     const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
-    uint32_t tcount = 0, sigcount = 0;
+    uint32_t tcount = 0, sigcount = 0, p2count = 0;
     int pending_u = -1;        // unit of the last pass-1 arrival still to resolve
     unsigned pending_old = 0;  // what the arrival counter held before it (thread 0)
     for (int seq = 0; ok; ++seq) {
@@ -603,35 +634,55 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
           ++tcount;
-          // online softmax partials, branch-free: re-base the running sum only
-          // when a logit exceeds the running reference by more than 2^20
-          if (it0 + kTile - 1 <= a.N - a.W) {
-            // every key of the tile is visible to every window row
-#pragma unroll
-            for (int c = 0; c < RH; ++c) {
-              const float x = __uint_as_float(rc[c]) * a.scale_log2;
-              const float dlt = (h * RH + c < a.R) ? x - m[c] : -INFINITY;
-              const bool up = dlt > 20.f;
-              const float ee = ex2(up ? -dlt : dlt);
-              z[c] = up ? fmaf(z[c], ee, 1.f) : z[c] + ee;
-              m[c] = up ? x : m[c];
-            }
-          } else {
-            // last tiles of the unit: window row j sees keys i <= N - W + j,
-            // and keys past N do not exist
-            const int vis_from = i - (a.N - a.W);  // row j sees key i iff j >= vis_from
+          // online softmax partials against a per-row reference m (the
+          // lane's first visible logit, 0 while there is none): z += 2^(x - m)
+          // with x - m kept at most 2^6 by re-basing the rare rows that jump
+          // above it.  Rows past R (padding, statistics) run unmasked; their
+          // partials are not kept.  x - m is computed in place in rc.
+          const bool full_vis = it0 + kTile - 1 <= a.N - a.W;  // every window row sees every key
+          const int vis_from = i - (a.N - a.W);                 // else row j sees key i iff j >= vis_from
+          if (t == 0) {
             int j = (h * RH) % a.W;
 #pragma unroll
             for (int c = 0; c < RH; ++c) {
-              const bool vis = (h * RH + c < a.R) && valid && j >= vis_from;
+              const bool vis = full_vis || (valid && j >= vis_from);
               if (++j == a.W) j = 0;
-              const float x = __uint_as_float(rc[c]) * a.scale_log2;
-              const float dlt = vis ? x - m[c] : -INFINITY;
-              const bool up = dlt > 20.f;
-              const float ee = ex2(up ? -dlt : dlt);
-              z[c] = up ? fmaf(z[c], ee, 1.f) : z[c] + ee;
-              m[c] = up ? x : m[c];
+              m[c] = vis ? __uint_as_float(rc[c]) * a.scale_log2 : 0.f;
+              z[c] = vis ? 1.f : 0.f;
             }
+          } else {
+            float mx = -INFINITY;
+            if (full_vis) {
+#pragma unroll
+              for (int c = 0; c < RH; ++c) {
+                const float dl = fmaf(__uint_as_float(rc[c]), a.scale_log2, -m[c]);
+                rc[c] = __float_as_uint(dl);
+                mx = fmaxf(mx, dl);
+              }
+            } else {
+              int j = (h * RH) % a.W;
+#pragma unroll
+              for (int c = 0; c < RH; ++c) {
+                const bool vis = valid && j >= vis_from;
+                if (++j == a.W) j = 0;
+                const float dl = vis ? fmaf(__uint_as_float(rc[c]), a.scale_log2, -m[c]) : -INFINITY;
+                rc[c] = __float_as_uint(dl);
+                mx = fmaxf(mx, dl);
+              }
+            }
+            if (mx > 64.f) {
+#pragma unroll
+              for (int c = 0; c < RH; ++c) {
+                const float dl = __uint_as_float(rc[c]);
+                if (dl > 20.f) {
+                  z[c] *= ex2(-dl);
+                  m[c] += dl;
+                  rc[c] = 0u;
+                }
+              }
+            }
+#pragma unroll
+            for (int c = 0; c < RH; ++c) z[c] += ex2(__uint_as_float(rc[c]));
           }
         }
         if (!ok) break;
@@ -639,14 +690,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // so that the RH rows' shuffles overlap
         float M[RH];
 #pragma unroll
-        for (int c = 0; c < RH; ++c) M[c] = m[c];
+        for (int c = 0; c < RH; ++c) M[c] = z[c] > 0.f ? m[c] : -INFINITY;  // lanes without a visible key do not count
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
           for (int c = 0; c < RH; ++c) M[c] = fmaxf(M[c], __shfl_xor_sync(0xffffffffu, M[c], o));
         }
 #pragma unroll
-        for (int c = 0; c < RH; ++c) z[c] = (m[c] == -INFINITY) ? 0.f : z[c] * ex2(m[c] - M[c]);
+        for (int c = 0; c < RH; ++c) z[c] = z[c] > 0.f ? z[c] * ex2(m[c] - M[c]) : 0.f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
@@ -708,7 +759,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < ntiles && ok; ++t) {
           const int i = i0 + t * kTile + kk;
           const bool valid = i < a.N;
-          const float n2 = (h == 0 && valid) ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;  // in flight early
           const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 14u))) break;
           tc_fence_after();
@@ -721,12 +771,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
           const uint32_t par = tcount & 1u;
           ++tcount;
+          float n2 = 0.f;
+          if (h == 0) {
+            // this key's squared norm from the key warps
+            const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
+            if (!(ok = wait_bar(&s.nfull[nb], nph, a, 15u))) break;
+            n2 = s.nbuf[nb][kk];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.nempty[nb]);
+          }
+          ++p2count;
+          // the lse of rows past R is +inf: their terms vanish without a mask
           float vp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < RH; ++c) {
-            const int rowi = h * RH + c;
-            if (rowi < a.R) vp[c & 3] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -lse[rowi]));
-          }
+          for (int c = 0; c < RH; ++c) vp[c & 3] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -lse[h * RH + c]));
           s.xch[par][h][kk] = (vp[0] + vp[1]) + (vp[2] + vp[3]);
           named_bar_sync(kEpiBar, kEpi);
           if (h == 0 && valid) {
@@ -752,7 +810,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               d2 = (dp[0] + dp[1]) + (dp[2] + dp[3]);
             }
             const float dEv = sqrtf(fmaxf(d2, 0.f));
-            const float cs = kmu * (1.f / fmaxf(sqrtf(n2), 1e-12f));
+            const float cs = kmu * rsqrtf(fmaxf(n2, 1e-24f));
             s_all += dEv;
             if (i < a.Tv) {
               mn = fminf(mn, dEv);
