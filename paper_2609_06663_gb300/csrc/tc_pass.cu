@@ -24,15 +24,17 @@
 // per-candidate arrays and per-chunk partial sums; finalisation, selection
 // and the gather of the kept rows run in the next launch (finalize_select.cu).
 //
-// Warp roles (384 threads, one CTA per SM): warp 0 takes tickets, resolves
+// Warp roles (512 threads, one CTA per SM): warp 0 takes tickets, resolves
 // dependencies (bounded spins on gpu-scope flags), loads the window queries
 // (TMA) and the unit statistics (bulk copy) and issues TMA loads of 32 KB key
-// tiles into a 4-stage ring; warp 1 issues the tcgen05 MMAs into up to four
-// TMEM accumulators (plus two for the sums); warps 2-3 (key warps) compute
-// the key norms and the sum weights of each pass-1 tile as soon as it lands,
-// so that a ring stage is freed without waiting for the softmax, and store
-// the norms for pass 2; warps 4-11 are the epilogue (one key per TMEM lane,
-// window rows split in two halves).  Every mbarrier wait and spin
+// tiles into a 5-stage ring; warp 1 issues the tcgen05 MMAs into up to four
+// TMEM accumulators (plus two for the sums); warps 12-15 (key warps, one key
+// per thread) compute the key norms and the sum weights of each pass-1 tile
+// as soon as it lands, so that a ring stage is freed without waiting for the
+// softmax, store the norms for pass 2 and hand them to the epilogue there;
+// warps 4-11 are the epilogue (one key per TMEM lane, window rows split in
+// two halves); warps 2-3 idle.  setmaxnreg gives the two epilogue
+// warpgroups 176 registers a thread and the others 80.  Every mbarrier wait and spin
 // is bounded: on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
 // gpu-wide abort flag, drains its own copies and MMAs, frees TMEM and exits.
 
@@ -50,9 +52,15 @@ using namespace ptx;
 
 constexpr int kIQ = 2;
 constexpr int kTile = 128;
-constexpr int kThreads = 384;
+constexpr int kThreads = 512;
 constexpr int kEpi = 256;
-constexpr int kEpiWarp0 = 4;          // first epilogue warp
+constexpr int kEpiWarp0 = 4;          // first epilogue warp (warps 4..11)
+constexpr int kKeyWarp0 = 12;         // first key warp (warps 12..15, one key per thread)
+constexpr int kKeyWarps = 4;
+constexpr uint32_t kRegsEpi = 176;    // registers a thread after the split: epilogue warpgroups
+constexpr uint32_t kRegsOther = 80;   // producer / MMA / key warpgroups
+static_assert(2 * 128 * kRegsEpi + 2 * 128 * kRegsOther == 65536, "register split must fit the launch's 512 x 128");
+static_assert(kRegsEpi % 8 == 0 && kRegsOther % 8 == 0 && kRegsOther >= 24 && kRegsEpi <= 256, "setmaxnreg range");
 constexpr int kNPMax = 128;
 constexpr uint32_t kTileBytes = kTile * kD * 2;
 constexpr uint32_t kTmemCols = 512;
@@ -286,12 +294,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], 3);   // 2 key warps + MMA commit
-      mbar_init(&s.wready[i], 2);  // 2 key warps
+      mbar_init(&s.empty[i], kKeyWarps + 1);  // key warps + MMA commit
+      mbar_init(&s.wready[i], kKeyWarps);
     }
     for (int i = 0; i < kIQ; ++i) {
       mbar_init(&s.item_full[i], 1);
-      mbar_init(&s.item_empty[i], 11);  // MMA commit + 8 epilogue warps + 2 key warps
+      mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps);  // MMA commit + 8 epilogue warps + key warps
       mbar_init(&s.qfull[i], 1);
     }
     for (int i = 0; i < 4; ++i) {
@@ -302,9 +310,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&s.sigma_full[i], 1);
       mbar_init(&s.sigma_empty[i], 4);
     }
-    for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], 2);  // 2 key warps
+    for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], kKeyWarps);
     for (int i = 0; i < kNB; ++i) {
-      mbar_init(&s.nfull[i], 2);   // 2 key warps
+      mbar_init(&s.nfull[i], kKeyWarps);
       mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the first row half
     }
     mbar_init(&s.drain, 1);
@@ -332,251 +340,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = s.tmem_base;
   bool ok = true;
 
-  if (warp == 0) {
-    // ------------------------------------------------ scheduler + TMA producer
-    int stage = 0;
-    uint32_t sphase = 0;
-    uint32_t used_bits = 0u, par_bits = 0u;  // per stage: loaded at least once / parity of loads
-    const uint64_t pol_keep = l2_policy_evict_last(), pol_drop = l2_policy_evict_first();
-    for (int seq = 0; ok;) {
-      int ticket = 0;
-      if (lane == 0) ticket = (int)atomicAdd(a.sync, 1u);
-      ticket = __shfl_sync(0xffffffffu, ticket, 0);
-      const Item it = decode(ticket, a);
-      if (!it.valid) continue;
-      const int slot = seq % kIQ;
-      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-      if (lane == 0) {
-        ok = wait_bar(&s.item_empty[slot], qphase ^ 1u, a, 1u);
-        if (ok && it.type == kP2) ok = wait_flag(a.sync + 4 + a.U + it.u, a, 2u);
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
-      if (!ok) break;
-      ItemDesc& d = s.desc[slot];
-      const int i0 = it.chunk * a.tiles_per_chunk * kTile;
-      const int ntiles = it.type == kExit ? 0 : min(a.tiles_per_chunk, (a.N - i0 + kTile - 1) / kTile);
-      if (lane == 0) {
-        d.type = it.type;
-        d.u = it.u;
-        d.chunk = it.chunk;
-        d.part = it.part;
-        d.i0 = i0;
-        d.ntiles = ntiles;
-      }
-      if (it.type == kP1 || it.type == kP2) {
-        // window queries by TMA (swizzled in flight); pass 2 also copies the
-        // unit statistics record
-        const uint32_t ust_bytes = (uint32_t)a.ustat_stride * 4u;
-        if (lane == 0) {
-          const int layer = it.u / a.h_kv, head = it.u % a.h_kv;
-          const int qrow = (layer * a.h_q + head * a.g) * a.W;
-          mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u + (it.type == kP2 ? ust_bytes : 0u));
-          tma_load_2d(s.qbuf[slot], &tmQ, &s.qfull[slot], 0, qrow);
-          tma_load_2d(s.qbuf[slot] + a.NP * 128, &tmQ, &s.qfull[slot], 64, qrow);
-          if (it.type == kP2) bulk_load(d.ust, a.ustat + (size_t)it.u * a.ustat_stride, ust_bytes, &s.qfull[slot]);
-          ok = wait_bar(&s.qfull[slot], qphase, a, 16u);
-        }
-        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
-        if (!ok) break;
-        if (it.type == kP2) build_stat_rows(s.qbuf[slot], a, d.ust, lane);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s.item_full[slot]);
-      ++seq;
-      if (it.type == kExit) break;
-      for (int t = 0; t < ntiles && ok; ++t) {
-        if (lane == 0) {
-          ok = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
-          if (ok) {
-            mbar_expect_tx(&s.full[stage], kTileBytes);
-            const int y = i0 + t * kTile;
-            // pass 1 keeps its keys in L2 for pass 2; pass 2 reads them for the last time
-            const uint64_t pol = it.type == kP1 ? pol_keep : pol_drop;
-            tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u, pol);
-            tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u, pol);
-            used_bits |= 1u << stage;
-            par_bits ^= 1u << stage;
-          }
-        }
-        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
-        if (++stage == kStages) {
-          stage = 0;
-          sphase ^= 1u;
-        }
-      }
-    }
-    if (!ok && lane == 0) {
-      // let this CTA's copies in flight land before its shared memory goes away
-      for (int st = 0; st < kStages; ++st)
-        if (used_bits & (1u << st)) {
-          const uint32_t last = ((par_bits >> st) & 1u) ^ 1u;  // parity of the last load's phase
-          const long long t0 = clock64();
-          while (!mbar_try_wait(&s.full[st], last) && clock64() - t0 < a.timeout_cycles) {
-          }
-        }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t sphase = 0, tcount = 0, sigcount = 0;
-      uint32_t wpar = 0u;  // per stage: parity of the next wready phase (pass-1 tiles only)
-      const uint32_t idesc_l = idesc_bf16(128, a.NP, false, false);
-      const uint32_t idesc_s = idesc_bf16(128, 16, true, false);
-      for (int seq = 0; ok; ++seq) {
-        const int slot = seq % kIQ;
-        const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-        if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 5u))) break;
-        const ItemDesc& d = s.desc[slot];
-        const int type = d.type, ntiles = d.ntiles;
-        if (type == kExit) break;
-        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
-        tc_fence_after();
-        const uint32_t qb = smem_u32(s.qbuf[slot]);
-        for (int t = 0; t < ntiles; ++t) {
-          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
-          if (!(ok = wait_bar(&s.full[stage], sphase, a, 6u))) break;
-          if (!(ok = wait_bar(&s.tmem_empty[b], tph ^ 1u, a, 7u))) break;
-          tc_fence_after();
-          const uint32_t kt = smem_u32(s.ktile[stage]);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint64_t ad = smem_desc(kt + (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32, 16, 1024, 2);
-            const uint64_t bd = smem_desc(qb + (kk >> 2) * (a.NP * 128) + (kk & 3) * 32, 16, 1024, 2);
-            mma_bf16(tmem + b * (uint32_t)a.NP, ad, bd, idesc_l, kk > 0 ? 1u : 0u);
-          }
-          mma_commit(&s.tmem_full[b]);
-          if (type == kP1) {
-            if (!(ok = wait_bar(&s.wready[stage], (wpar >> stage) & 1u, a, 8u))) break;
-            wpar ^= 1u << stage;
-            const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
-            if (t == 0 && !(ok = wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u))) break;
-            tc_fence_after();
-            const uint32_t wb = smem_u32(s.wbuf[stage]);
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              // A = key tile viewed MN-major (d contiguous): 16 keys per step
-              const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
-              const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
-              mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
-            }
-          }
-          mma_commit(&s.empty[stage]);
-          if (type == kP1 && t == ntiles - 1) {
-            mma_commit(&s.sigma_full[sigcount & 1u]);
-            ++sigcount;
-          }
-          ++tcount;
-          if (++stage == kStages) {
-            stage = 0;
-            sphase ^= 1u;
-          }
-        }
-        if (!ok) break;
-        mma_commit(&s.item_empty[slot]);
-      }
-      if (!ok) {
-        mma_commit(&s.drain);
-        const long long t0 = clock64();
-        while (!mbar_try_wait(&s.drain, 0u) && clock64() - t0 < a.timeout_cycles) {
-        }
-      }
-    }
-  } else if (warp < kEpiWarp0) {
-    // ------------------------------------------------ key warps (2..3)
-    const int tk = threadIdx.x - 64;  // 0..63: keys tk and tk + 64 of each tile
-    int stage = 0;
-    uint32_t sphase = 0, p2count = 0;
-    for (int seq = 0; ok; ++seq) {
-      const int slot = seq % kIQ;
-      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-      if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 20u))) break;
-      const ItemDesc& d = s.desc[slot];
-      const int type = d.type, ntiles = d.ntiles, i0 = d.i0, u = d.u;
-      if (type == kExit) break;
-      for (int t = 0; t < ntiles && ok; ++t) {
-        if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
-        if (type == kP1) {
-          // squared norms of this thread's two keys (packed fp32 pairs), kept
-          // for pass 2, and the sum weights w = 1/||k|| in three bf16 terms
-          float n2v[2];
-#pragma unroll
-          for (int q2 = 0; q2 < 2; ++q2) {
-            const int kk = tk + 64 * q2;
-            uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-            for (int hb = 0; hb < 2; ++hb) {
-              const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
-#pragma unroll
-              for (int c = 0; c < 8; ++c) {
-                const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
-                const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                for (int t2 = 0; t2 < 4; ++t2) {
-                  const uint64_t x = pack_f32x2(__uint_as_float(w4[t2] << 16), __uint_as_float(w4[t2] & 0xffff0000u));
-                  acc[t2] = ffma2(x, x, acc[t2]);
-                }
-              }
-            }
-            n2v[q2] = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
-                      ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
-#pragma unroll
-          for (int q2 = 0; q2 < 2; ++q2) {
-            const int kk = tk + 64 * q2;
-            const int i = i0 + t * kTile + kk;
-            const bool valid = i < a.N;
-            if (valid) a.norm2[(size_t)u * a.N + i] = n2v[q2];
-            const float w = valid ? rsqrtf(fmaxf(n2v[q2], 1e-24f)) : 0.f;
-            const __nv_bfloat16 whi = __float2bfloat16_rn(w);
-            const float r1 = w - __bfloat162float(whi);
-            const __nv_bfloat16 wmid = __float2bfloat16_rn(r1);
-            const __nv_bfloat16 wlo = __float2bfloat16_rn(r1 - __bfloat162float(wmid));
-            uint8_t* base = s.wbuf[stage] + (kk >> 6) * 2048 + (kk & 7) * 2;
-            const int j = (kk & 63) >> 3;
-            *reinterpret_cast<__nv_bfloat16*>(base + sw128(1, j)) = whi;
-            *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
-            *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.wready[stage]);
-        } else {
-          // pass 2: the keys are only needed by the MMA; the norms pass 1
-          // stored go to the epilogue through shared memory
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.empty[stage]);
-          const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
-          ++p2count;
-          const int ia = i0 + t * kTile + tk, ib = ia + 64;
-          const float na = ia < a.N ? __ldcg(a.norm2 + (size_t)u * a.N + ia) : 0.f;
-          const float nbv = ib < a.N ? __ldcg(a.norm2 + (size_t)u * a.N + ib) : 0.f;
-          if (!(ok = wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u))) break;
-          s.nbuf[nb][tk] = na;
-          s.nbuf[nb][tk + 64] = nbv;
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.nfull[nb]);
-        }
-        if (++stage == kStages) {
-          stage = 0;
-          sphase ^= 1u;
-        }
-      }
-      if (!ok) break;
-      // publish this item's key norms at gpu scope before the epilogue counts
-      // the item as arrived (the fence is cumulative over the warp's stores
-      // ordered before it by __syncwarp)
-      __syncwarp();
-      if (lane == 0) {
-        if (type == kP1) __threadfence();
-        mbar_arrive(&s.kpub[slot]);
-        mbar_arrive(&s.item_empty[slot]);
-      }
-    }
-  } else {
+  if (warp >= kEpiWarp0 && warp < kKeyWarp0) {
+    // register split: the two epilogue warpgroups take the registers the
+    // other two give back
+    reg_alloc<kRegsEpi>();
     // ------------------------------------------------ epilogue (warps 4..11)
     const int e = warp - kEpiWarp0, q = warp & 3, h = e >> 2;
     const int kk = 32 * q + lane;  // key row within a tile = TMEM lane
@@ -860,6 +627,241 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.item_empty[slot]);
     }
+  } else {
+    reg_dealloc<kRegsOther>();
+  if (warp == 0) {
+    // ------------------------------------------------ scheduler + TMA producer
+    int stage = 0;
+    uint32_t sphase = 0;
+    uint32_t used_bits = 0u, par_bits = 0u;  // per stage: loaded at least once / parity of loads
+    const uint64_t pol_keep = l2_policy_evict_last(), pol_drop = l2_policy_evict_first();
+    for (int seq = 0; ok;) {
+      int ticket = 0;
+      if (lane == 0) ticket = (int)atomicAdd(a.sync, 1u);
+      ticket = __shfl_sync(0xffffffffu, ticket, 0);
+      const Item it = decode(ticket, a);
+      if (!it.valid) continue;
+      const int slot = seq % kIQ;
+      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+      if (lane == 0) {
+        ok = wait_bar(&s.item_empty[slot], qphase ^ 1u, a, 1u);
+        if (ok && it.type == kP2) ok = wait_flag(a.sync + 4 + a.U + it.u, a, 2u);
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+      if (!ok) break;
+      ItemDesc& d = s.desc[slot];
+      const int i0 = it.chunk * a.tiles_per_chunk * kTile;
+      const int ntiles = it.type == kExit ? 0 : min(a.tiles_per_chunk, (a.N - i0 + kTile - 1) / kTile);
+      if (lane == 0) {
+        d.type = it.type;
+        d.u = it.u;
+        d.chunk = it.chunk;
+        d.part = it.part;
+        d.i0 = i0;
+        d.ntiles = ntiles;
+      }
+      if (it.type == kP1 || it.type == kP2) {
+        // window queries by TMA (swizzled in flight); pass 2 also copies the
+        // unit statistics record
+        const uint32_t ust_bytes = (uint32_t)a.ustat_stride * 4u;
+        if (lane == 0) {
+          const int layer = it.u / a.h_kv, head = it.u % a.h_kv;
+          const int qrow = (layer * a.h_q + head * a.g) * a.W;
+          mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u + (it.type == kP2 ? ust_bytes : 0u));
+          tma_load_2d(s.qbuf[slot], &tmQ, &s.qfull[slot], 0, qrow);
+          tma_load_2d(s.qbuf[slot] + a.NP * 128, &tmQ, &s.qfull[slot], 64, qrow);
+          if (it.type == kP2) bulk_load(d.ust, a.ustat + (size_t)it.u * a.ustat_stride, ust_bytes, &s.qfull[slot]);
+          ok = wait_bar(&s.qfull[slot], qphase, a, 16u);
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        if (!ok) break;
+        if (it.type == kP2) build_stat_rows(s.qbuf[slot], a, d.ust, lane);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.item_full[slot]);
+      ++seq;
+      if (it.type == kExit) break;
+      for (int t = 0; t < ntiles && ok; ++t) {
+        if (lane == 0) {
+          ok = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
+          if (ok) {
+            mbar_expect_tx(&s.full[stage], kTileBytes);
+            const int y = i0 + t * kTile;
+            // pass 1 keeps its keys in L2 for pass 2; pass 2 reads them for the last time
+            const uint64_t pol = it.type == kP1 ? pol_keep : pol_drop;
+            tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u, pol);
+            tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u, pol);
+            used_bits |= 1u << stage;
+            par_bits ^= 1u << stage;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        if (++stage == kStages) {
+          stage = 0;
+          sphase ^= 1u;
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      // let this CTA's copies in flight land before its shared memory goes away
+      for (int st = 0; st < kStages; ++st)
+        if (used_bits & (1u << st)) {
+          const uint32_t last = ((par_bits >> st) & 1u) ^ 1u;  // parity of the last load's phase
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&s.full[st], last) && clock64() - t0 < a.timeout_cycles) {
+          }
+        }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t sphase = 0, tcount = 0, sigcount = 0;
+      uint32_t wpar = 0u;  // per stage: parity of the next wready phase (pass-1 tiles only)
+      const uint32_t idesc_l = idesc_bf16(128, a.NP, false, false);
+      const uint32_t idesc_s = idesc_bf16(128, 16, true, false);
+      for (int seq = 0; ok; ++seq) {
+        const int slot = seq % kIQ;
+        const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+        if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 5u))) break;
+        const ItemDesc& d = s.desc[slot];
+        const int type = d.type, ntiles = d.ntiles;
+        if (type == kExit) break;
+        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
+        tc_fence_after();
+        const uint32_t qb = smem_u32(s.qbuf[slot]);
+        for (int t = 0; t < ntiles; ++t) {
+          const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
+          if (!(ok = wait_bar(&s.full[stage], sphase, a, 6u))) break;
+          if (!(ok = wait_bar(&s.tmem_empty[b], tph ^ 1u, a, 7u))) break;
+          tc_fence_after();
+          const uint32_t kt = smem_u32(s.ktile[stage]);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint64_t ad = smem_desc(kt + (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32, 16, 1024, 2);
+            const uint64_t bd = smem_desc(qb + (kk >> 2) * (a.NP * 128) + (kk & 3) * 32, 16, 1024, 2);
+            mma_bf16(tmem + b * (uint32_t)a.NP, ad, bd, idesc_l, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&s.tmem_full[b]);
+          if (type == kP1) {
+            if (!(ok = wait_bar(&s.wready[stage], (wpar >> stage) & 1u, a, 8u))) break;
+            wpar ^= 1u << stage;
+            const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+            if (t == 0 && !(ok = wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u))) break;
+            tc_fence_after();
+            const uint32_t wb = smem_u32(s.wbuf[stage]);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              // A = key tile viewed MN-major (d contiguous): 16 keys per step
+              const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
+              const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
+              mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
+            }
+          }
+          mma_commit(&s.empty[stage]);
+          if (type == kP1 && t == ntiles - 1) {
+            mma_commit(&s.sigma_full[sigcount & 1u]);
+            ++sigcount;
+          }
+          ++tcount;
+          if (++stage == kStages) {
+            stage = 0;
+            sphase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit(&s.item_empty[slot]);
+      }
+      if (!ok) {
+        mma_commit(&s.drain);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(&s.drain, 0u) && clock64() - t0 < a.timeout_cycles) {
+        }
+      }
+    }
+  } else if (warp >= kKeyWarp0) {
+    // ------------------------------------------------ key warps (12..15)
+    const int kk = threadIdx.x - 32 * kKeyWarp0;  // 0..127: this thread's key row of each tile
+    int stage = 0;
+    uint32_t sphase = 0, p2count = 0;
+    for (int seq = 0; ok; ++seq) {
+      const int slot = seq % kIQ;
+      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+      if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 20u))) break;
+      const ItemDesc& d = s.desc[slot];
+      const int type = d.type, ntiles = d.ntiles, i0 = d.i0, u = d.u;
+      if (type == kExit) break;
+      for (int t = 0; t < ntiles && ok; ++t) {
+        if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
+        const int i = i0 + t * kTile + kk;
+        const bool valid = i < a.N;
+        if (type == kP1) {
+          // squared norm of this thread's key (packed fp32 pairs), kept for
+          // pass 2, and the sum weights w = 1/||k|| in three bf16 terms
+          uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+          for (int hb = 0; hb < 2; ++hb) {
+            const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
+              const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+              for (int t2 = 0; t2 < 4; ++t2) {
+                const uint64_t x = pack_f32x2(__uint_as_float(w4[t2] << 16), __uint_as_float(w4[t2] & 0xffff0000u));
+                acc[t2] = ffma2(x, x, acc[t2]);
+              }
+            }
+          }
+          const float n2 = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
+                           ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
+          if (valid) a.norm2[(size_t)u * a.N + i] = n2;
+          const float w = valid ? rsqrtf(fmaxf(n2, 1e-24f)) : 0.f;
+          const __nv_bfloat16 whi = __float2bfloat16_rn(w);
+          const float r1 = w - __bfloat162float(whi);
+          const __nv_bfloat16 wmid = __float2bfloat16_rn(r1);
+          const __nv_bfloat16 wlo = __float2bfloat16_rn(r1 - __bfloat162float(wmid));
+          uint8_t* base = s.wbuf[stage] + (kk >> 6) * 2048 + (kk & 7) * 2;
+          const int j = (kk & 63) >> 3;
+          *reinterpret_cast<__nv_bfloat16*>(base + sw128(1, j)) = whi;
+          *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
+          *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.wready[stage]);
+        } else {
+          // pass 2: the keys are only needed by the MMA; the norms pass 1
+          // stored go to the epilogue through shared memory
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.empty[stage]);
+          const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
+          ++p2count;
+          const float n2 = valid ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;
+          if (!(ok = wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u))) break;
+          s.nbuf[nb][kk] = n2;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.nfull[nb]);
+        }
+        if (++stage == kStages) {
+          stage = 0;
+          sphase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      // publish this item's key norms at gpu scope before the epilogue counts
+      // the item as arrived (the fence is cumulative over the warp's stores
+      // ordered before it by __syncwarp)
+      __syncwarp();
+      if (lane == 0) {
+        if (type == kP1) __threadfence();
+        mbar_arrive(&s.kpub[slot]);
+        mbar_arrive(&s.item_empty[slot]);
+      }
+    }
+    }
   }
 
   tc_fence_before();
@@ -878,7 +880,13 @@ cudaError_t launch_rh(const CUtensorMap& tm, const CUtensorMap& tq, const TcArgs
   const size_t smem = sizeof(Smem<RH>) + 1024;
   const int rh_i = RH == 8 ? 0 : RH == 16 ? 1 : RH == 32 ? 2 : 3;
   if (!g_attr_set[dev][rh_i]) {
-    cudaError_t e = cudaFuncSetAttribute(tc_evict_kernel<RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    // the warpgroups' register split needs the launch to give every thread
+    // 65536 / kThreads registers; refuse to launch otherwise
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, tc_evict_kernel<RH>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs * kThreads < 2 * 128 * (int)(kRegsEpi + kRegsOther)) return cudaErrorInvalidConfiguration;
+    e = cudaFuncSetAttribute(tc_evict_kernel<RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     g_attr_set[dev][rh_i] = true;
   }
