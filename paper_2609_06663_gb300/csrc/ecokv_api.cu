@@ -29,7 +29,7 @@ Layout make_layout(const ecokv_params& p, int chunk) {
   L.Tv = p.n - p.window;
   L.chunk = chunk;
   L.nchunks = (p.n + chunk - 1) / chunk;
-  L.p1_stride = 2 * L.R + 2 * kD;
+  L.p1_stride = 2 * ((L.R + 3) & ~3) + 2 * kD;
   L.ustat_stride = (ustat_lse() + L.R + 3) & ~3;
   const size_t U = (size_t)L.U;
   size_t off = 0;

@@ -45,6 +45,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
@@ -118,6 +121,19 @@ __device__ __forceinline__ uint64_t pack_f32x2(float lo, float hi) {
 }
 __device__ __forceinline__ float f32x2_lo(uint64_t v) { return __uint_as_float((uint32_t)v); }
 __device__ __forceinline__ float f32x2_hi(uint64_t v) { return __uint_as_float((uint32_t)(v >> 32)); }
+
+// a0 += lo(w)^2, a1 += hi(w)^2 for the two bf16 halves of w, each a single
+// fp32 fused multiply-add of the exactly widened values (sm_100+ mixed fma).
+__device__ __forceinline__ void sq_acc_bf16x2(uint32_t w, float& a0, float& a1) {
+  asm("{\n"
+      " .reg .b16 lo, hi;\n"
+      " mov.b32 {lo, hi}, %2;\n"
+      " fma.rn.f32.bf16 %0, lo, lo, %0;\n"
+      " fma.rn.f32.bf16 %1, hi, hi, %1;\n"
+      "}\n"
+      : "+f"(a0), "+f"(a1)
+      : "r"(w));
+}
 
 // ---------------------------------------------------------------- tcgen05
 __device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {

@@ -89,29 +89,26 @@ struct __align__(1024) Smem {
   uint8_t qbuf[kIQ][kQB < 1024 ? 1024 : kQB];   // B operand, 2 boxes [NP rows x 64 d]
   uint8_t wbuf[kS][4096];                       // sum weights: 2 boxes [16 rows x 64 keys]; rows 1, w_hi, w_mid, w_lo
   ItemDesc desc[kIQ];
-  float xch[2][2][kTile];                       // [tile parity][row half][key]
+  float xch[kNB][kTile];                        // pass-2 vote of the first row half, per key
   float red[8][RH][2];                          // [epilogue warp][row][max, sum]
-  float red6[8][8];                             // [epilogue warp][pass-2 partial]
-  float shf[64];
+  float red6[4][8];                             // [second-half warp][pass-2 partial]
   uint64_t full[kS], empty[kS], wready[kS];
   uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
   uint64_t tmem_full[4], tmem_empty[4];
   uint64_t sigma_full[2], sigma_empty[2], drain;
   float nbuf[kNB][kTile];                        // pass-2 squared key norms, key warps -> epilogue
   uint64_t nfull[kNB], nempty[kNB];
-  uint64_t kpub[kIQ];  // key warps have published this item's key norms (gpu scope)
+  uint64_t xfull[kNB], xempty[kNB];             // first row half -> second row half, per pass-2 tile
+  uint64_t kpub[kIQ];    // key warps have published this item's key norms (gpu scope)
+  uint64_t p1done[kIQ];  // the epilogue has written this pass-1 item's partials
   uint32_t tmem_base;
-  int flag_last;
+  int epi_abort;         // an epilogue warp gave up a wait (read after a named barrier)
 };
 
 static_assert(sizeof(Smem<8>) + 1024 <= 232448 && sizeof(Smem<16>) + 1024 <= 232448 &&
                   sizeof(Smem<32>) + 1024 <= 232448 && sizeof(Smem<64>) + 1024 <= 232448,
               "shared-memory plan exceeds the 227 KB per-CTA limit");
 static_assert(sizeof(ItemDesc) % 16 == 0 && offsetof(ItemDesc, ust) % 16 == 0, "bulk-copy target alignment");
-
-struct EpiSync {
-  __device__ __forceinline__ static void sync() { named_bar_sync(kEpiBar, kEpi); }
-};
 
 __device__ __forceinline__ unsigned* abort_flag(const TcArgs& a) { return a.sync + 1; }
 
@@ -187,9 +184,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// Pass-2 rows of the B operand (128-byte-swizzled, K-major): rows R4..R4+2
-// hold kbar split into three bf16 terms (hi, mid, lo), rows R4+3, R4+4 hold
-// mu_hi and mu_lo, all from the unit statistics copy; the window queries in
+// Pass-2 rows of the B operand (128-byte-swizzled, K-major): rows NP-8..NP-6
+// hold kbar split into three bf16 terms (hi, mid, lo), rows NP-5, NP-4 hold
+// mu_hi and mu_lo, all from the unit statistics copy (the last eight columns
+// of the accumulator belong to the second row half); the window queries in
 // rows 0..R-1 arrive by TMA.  Run by the 32 lanes of warp 0.
 __device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, float* ust, int lane) {
   // rows past the window rows (padding and the statistics rows) get an
@@ -210,74 +208,113 @@ __device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, float* ust, int la
     }
     const uint4 val = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
                                  pack_bf16x2(o[6], o[7]));
-    *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(a.R4 + which, j & 7)) = val;
+    *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(a.NP - 8 + which, j & 7)) = val;
   }
 }
 
-// Fold every chunk's pass-1 partials of unit u into its statistics record.
-// Threads [0, R) take one window row each (chunk maxima, then the rescaled
-// exp-sums), threads [128, 256) one key dimension each (sums of k and of
-// k/||k||); loads go out in batches of 16 so the L2 latency is paid a few
-// times per unit rather than once per chunk.
-__device__ void unit_reduce(const TcArgs& a, int u, float* shf, int tid) {
-  __threadfence();
-  constexpr int kB = 16;
-  const float* base = a.p1part + (size_t)u * a.nchunks * a.p1_stride;
-  float* us = a.ustat + (size_t)u * a.ustat_stride;
+// Fold every chunk's pass-1 partials of unit u into its statistics record,
+// one warp: lane l sums key dimensions 4l..4l+3 (16-byte loads) and combines
+// the (max, sum) pairs of window rows l, l + 32, ... online.  Loads go out in
+// batches so that the L2 latency is paid a few times per unit.  Chunk record:
+// [sum k (d)] [sum k/||k|| (d)] [row max (R4)] [row sum (R4)].
+__device__ void unit_reduce_warp(const TcArgs& a, int u, int lane) {
   const int nch = a.nchunks;
-  float kb = 0.f, mu = 0.f;
-  if (tid < a.R) {
-    const int r = tid;
-    float M = -INFINITY;
-    for (int c0 = 0; c0 < nch; c0 += kB) {
-      float mv[kB];
+  const float* base = a.p1part + (size_t)u * nch * a.p1_stride;
+  float* us = a.ustat + (size_t)u * a.ustat_stride;
+  constexpr int kB = 8;
+  float4 sk = make_float4(0.f, 0.f, 0.f, 0.f), sh = sk;
+  for (int c0 = 0; c0 < nch; c0 += kB) {
+    float4 kv[kB], hv[kB];
 #pragma unroll
-      for (int j = 0; j < kB; ++j) mv[j] = c0 + j < nch ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + r) : -INFINITY;
-#pragma unroll
-      for (int j = 0; j < kB; ++j) M = fmaxf(M, mv[j]);
+    for (int j = 0; j < kB; ++j) {
+      const float4* p = reinterpret_cast<const float4*>(base + (size_t)min(c0 + j, nch - 1) * a.p1_stride);
+      kv[j] = __ldcg(p + lane);
+      hv[j] = __ldcg(p + kD / 4 + lane);
     }
-    float Z = 0.f;
-    for (int c0 = 0; c0 < nch; c0 += kB) {
-      float mv[kB], zv[kB];
 #pragma unroll
-      for (int j = 0; j < kB; ++j) {
-        const bool in = c0 + j < nch;
-        mv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + r) : -INFINITY;
-        zv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + a.R + r) : 0.f;
+    for (int j = 0; j < kB; ++j)
+      if (c0 + j < nch) {
+        sk.x += kv[j].x; sk.y += kv[j].y; sk.z += kv[j].z; sk.w += kv[j].w;
+        sh.x += hv[j].x; sh.y += hv[j].y; sh.z += hv[j].z; sh.w += hv[j].w;
       }
-#pragma unroll
-      for (int j = 0; j < kB; ++j)
-        if (mv[j] != -INFINITY) Z += zv[j] * ex2(mv[j] - M);
-    }
-    us[ustat_lse() + r] = M + log2f(Z);
-  } else if (tid >= 128) {
-    const int dd = tid - 128;
-    float sk = 0.f, skh = 0.f;
-    for (int c0 = 0; c0 < nch; c0 += kB) {
-      float kv[kB], hv[kB];
-#pragma unroll
-      for (int j = 0; j < kB; ++j) {
-        const bool in = c0 + j < nch;
-        kv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + 2 * a.R + dd) : 0.f;
-        hv[j] = in ? __ldcg(base + (size_t)(c0 + j) * a.p1_stride + 2 * a.R + kD + dd) : 0.f;
-      }
-#pragma unroll
-      for (int j = 0; j < kB; ++j) {
-        sk += kv[j];
-        skh += hv[j];
-      }
-    }
-    const float inv_n = 1.f / (float)a.N;
-    kb = sk * inv_n;
-    mu = skh * inv_n;
-    us[ustat_kbar() + dd] = kb;
-    us[ustat_mu() + dd] = mu;
   }
-  const float ksq = group_reduce<Op::Sum, EpiSync>(kb * kb, shf, tid, kEpi);
-  const float msq = group_reduce<Op::Sum, EpiSync>(mu * mu, shf, tid, kEpi);
-  if (tid == 0) {
+  const float inv_n = 1.f / (float)a.N;
+  const float4 kb = make_float4(sk.x * inv_n, sk.y * inv_n, sk.z * inv_n, sk.w * inv_n);
+  const float4 mu = make_float4(sh.x * inv_n, sh.y * inv_n, sh.z * inv_n, sh.w * inv_n);
+  reinterpret_cast<float4*>(us + ustat_kbar())[lane] = kb;
+  reinterpret_cast<float4*>(us + ustat_mu())[lane] = mu;
+  float ksq = (kb.x * kb.x + kb.y * kb.y) + (kb.z * kb.z + kb.w * kb.w);
+  float msq = (mu.x * mu.x + mu.y * mu.y) + (mu.z * mu.z + mu.w * mu.w);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ksq += __shfl_xor_sync(0xffffffffu, ksq, o);
+    msq += __shfl_xor_sync(0xffffffffu, msq, o);
+  }
+  if (lane == 0) {
     us[ustat_ksq()] = ksq;
     us[ustat_musq()] = msq;
+  }
+  for (int r = lane; r < a.R; r += 32) {
+    float M = -INFINITY, Z = 0.f;
+    constexpr int kR = 16;
+    for (int c0 = 0; c0 < nch; c0 += kR) {
+      float mv[kR], zv[kR];
+#pragma unroll
+      for (int j = 0; j < kR; ++j) {
+        const float* p = base + (size_t)min(c0 + j, nch - 1) * a.p1_stride + 2 * kD;
+        mv[j] = __ldcg(p + r);
+        zv[j] = c0 + j < nch ? __ldcg(p + a.R4 + r) : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < kR; ++j)
+        if (zv[j] > 0.f) {
+          const float Mn = fmaxf(M, mv[j]);
+          Z = Z * ex2(M - Mn) + zv[j] * ex2(mv[j] - Mn);
+          M = Mn;
+        }
+    }
+    us[ustat_lse() + r] = M + log2f(Z);
+  }
+}
+
+// Joint (max, sum) of partial softmax sums: (m1, z1) + (m2, z2) with z
+// relative to 2^m; an empty pair has m = -inf, z = 0.
+__device__ __forceinline__ void combine_maxsum(float& m, float& z, float m2, float z2) {
+  const float M = fmaxf(m, m2);
+  const float Ms = M == -INFINITY ? 0.f : M;
+  z = z * ex2(m - Ms) + z2 * ex2(m2 - Ms);
+  m = M;
+}
+
+// Reduce-scatter of RH (max, sum) rows over the 32 lanes of a warp: each
+// step exchanges half of the remaining rows with the partner lane, so lane l
+// ends with row (l >> shift) * per + j in m[j], z[j] (shift = 0, 1, 2 for
+// RH = 32 (or more), 16, 8; per = RH / 32 rows when RH > 32); lanes that share
+// a row hold the same value.
+template <int RH>
+__device__ __forceinline__ void warp_reduce_scatter_maxsum(float (&m)[RH], float (&z)[RH], int lane) {
+  int n = RH;
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    if (n > 1 && (RH > 32 || n > 1)) {
+      const bool up = (lane & o) != 0;
+      const int hf = n / 2;
+#pragma unroll
+      for (int j = 0; j < RH / 2; ++j) {
+        if (j < hf) {
+          const float km = up ? m[j + hf] : m[j], kz = up ? z[j + hf] : z[j];
+          const float sm = up ? m[j] : m[j + hf], sz = up ? z[j] : z[j + hf];
+          const float rm = __shfl_xor_sync(0xffffffffu, sm, o), rz = __shfl_xor_sync(0xffffffffu, sz, o);
+          m[j] = km;
+          z[j] = kz;
+          combine_maxsum(m[j], z[j], rm, rz);
+        }
+      }
+      n = hf;
+    } else {
+      const float rm = __shfl_xor_sync(0xffffffffu, m[0], o), rz = __shfl_xor_sync(0xffffffffu, z[0], o);
+      combine_maxsum(m[0], z[0], rm, rz);
+    }
   }
 }
 
@@ -299,7 +336,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kIQ; ++i) {
       mbar_init(&s.item_full[i], 1);
-      mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps);  // MMA commit + 8 epilogue warps + key warps
+      mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps + 1);  // MMA commit + epilogue + key warps + stats warp
+      mbar_init(&s.p1done[i], 8);
       mbar_init(&s.qfull[i], 1);
     }
     for (int i = 0; i < 4; ++i) {
@@ -313,8 +351,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], kKeyWarps);
     for (int i = 0; i < kNB; ++i) {
       mbar_init(&s.nfull[i], kKeyWarps);
-      mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the first row half
+      mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the second row half
+      mbar_init(&s.xfull[i], 4);   // first row half
+      mbar_init(&s.xempty[i], 4);  // second row half
     }
+    s.epi_abort = 0;
     mbar_init(&s.drain, 1);
     fence_mbar_init();
   }
@@ -345,35 +386,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     // other two give back
     reg_alloc<kRegsEpi>();
     // ------------------------------------------------ epilogue (warps 4..11)
+    // Named barriers among the eight warps sit only at item boundaries and are
+    // reached by every warp; a warp that gives up a wait marks epi_abort and
+    // all of them leave together after the next barrier.
     const int e = warp - kEpiWarp0, q = warp & 3, h = e >> 2;
     const int kk = 32 * q + lane;  // key row within a tile = TMEM lane
     const int tid = threadIdx.x - 32 * kEpiWarp0;
     const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
-    uint32_t tcount = 0, sigcount = 0, p2count = 0;
-    int pending_u = -1;        // unit of the last pass-1 arrival still to resolve
-    unsigned pending_old = 0;  // what the arrival counter held before it (thread 0)
-    for (int seq = 0; ok; ++seq) {
-      if (pending_u >= 0) {
-        // the pass-1 arrival of the previous item: the last of its unit folds
-        // the chunk partials into the unit statistics
-        if (tid == 0) s.flag_last = pending_old == (unsigned)(a.nchunks - 1);
-        named_bar_sync(kEpiBar, kEpi);
-        const bool last = s.flag_last != 0;
-        named_bar_sync(kEpiBar, kEpi);
-        if (last) {
-          unit_reduce(a, pending_u, s.shf, tid);
-          __threadfence();
-          named_bar_sync(kEpiBar, kEpi);
-          if (tid == 0) {
-            __threadfence();
-            st_release(a.sync + 4 + a.U + pending_u, 1u);
-          }
-        }
-        pending_u = -1;
-      }
+    const uint32_t bmask = (1u << nbuf_log) - 1u;
+    uint32_t tcount = 0, pcount = 0;
+    auto epi_sync = [&]() -> bool {
+      if (!ok) s.epi_abort = 1;
+      named_bar_sync(kEpiBar, kEpi);
+      return s.epi_abort == 0;
+    };
+    for (int seq = 0;; ++seq) {
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-      if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 10u))) break;
+      ok = __all_sync(0xffffffffu, wait_bar(&s.item_full[slot], qphase, a, 10u));
+      if (!epi_sync()) {
+        ok = false;
+        break;
+      }
       const ItemDesc& d = s.desc[slot];
       const int type = d.type;
       if (type == kExit) break;
@@ -383,16 +417,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         float m[RH], z[RH];
 #pragma unroll
         for (int c = 0; c < RH; ++c) {
-          m[c] = -INFINITY;
+          m[c] = 0.f;
           z[c] = 0.f;
         }
-        const uint32_t bmask = (1u << nbuf_log) - 1u;
         for (int t = 0; t < ntiles && ok; ++t) {
           const int it0 = i0 + t * kTile;
           const int i = it0 + kk;
           const bool valid = i < a.N;
           const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
-          if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 12u))) break;
+          if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.tmem_full[b], tph, a, 12u)))) break;
           tc_fence_after();
           uint32_t rc[RH];
           tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), rc);
@@ -452,32 +485,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < RH; ++c) z[c] += ex2(__uint_as_float(rc[c]));
           }
         }
-        if (!ok) break;
-        // item end: per-row (max, sum) over the 32 keys of the warp, step-major
-        // so that the RH rows' shuffles overlap
-        float M[RH];
+        // item end: per-row (max, sum) over the 32 keys of the warp by a
+        // reduce-scatter (31 shuffle pairs instead of 5 per row)
 #pragma unroll
-        for (int c = 0; c < RH; ++c) M[c] = z[c] > 0.f ? m[c] : -INFINITY;  // lanes without a visible key do not count
+        for (int c = 0; c < RH; ++c) m[c] = z[c] > 0.f ? m[c] : -INFINITY;  // lanes without a visible key do not count
+        warp_reduce_scatter_maxsum<RH>(m, z, lane);
+        constexpr int kShift = RH >= 32 ? 0 : (RH == 16 ? 1 : 2);  // lanes sharing a row after the scatter
+        constexpr int kPer = RH > 32 ? RH / 32 : 1;                  // rows a lane holds
+        if ((lane & ((1 << kShift) - 1)) == 0) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-#pragma unroll
-          for (int c = 0; c < RH; ++c) M[c] = fmaxf(M[c], __shfl_xor_sync(0xffffffffu, M[c], o));
-        }
-#pragma unroll
-        for (int c = 0; c < RH; ++c) z[c] = z[c] > 0.f ? z[c] * ex2(m[c] - M[c]) : 0.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-#pragma unroll
-          for (int c = 0; c < RH; ++c) z[c] += __shfl_xor_sync(0xffffffffu, z[c], o);
-        }
-        if (lane == 0) {
-#pragma unroll
-          for (int c = 0; c < RH; ++c) {
-            s.red[e][c][0] = M[c];
-            s.red[e][c][1] = z[c];
+          for (int j = 0; j < kPer; ++j) {
+            const int row = (lane >> kShift) * kPer + j;
+            s.red[e][row][0] = m[j];
+            s.red[e][row][1] = z[j];
           }
         }
-        named_bar_sync(kEpiBar, kEpi);
+        if (!epi_sync()) {
+          ok = false;
+          break;
+        }
         float* part = a.p1part + ((size_t)u * a.nchunks + chunk) * a.p1_stride;
         if (tid < a.R) {
           const int hh = tid / RH, c = tid % RH;
@@ -490,76 +516,57 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float mm = s.red[4 * hh + w4][c][0];
             if (mm != -INFINITY) Z += s.red[4 * hh + w4][c][1] * ex2(mm - Mx);
           }
-          part[tid] = Mx;
-          part[a.R + tid] = Z;
+          part[2 * kD + tid] = Mx;
+          part[2 * kD + a.R4 + tid] = Z;
         }
-        // chunk sums of k and k/||k|| from the weight MMA (TMEM lane = dimension)
-        if (h == 0) {
-          const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
-          if (!(ok = wait_bar(&s.sigma_full[sb], sph, a, 13u))) break;
-          tc_fence_after();
-          uint32_t v[4];
-          tmem_ld_x4(tl + kSigmaCol + 16u * sb, v);
-          tmem_wait_ld();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.sigma_empty[sb]);
-          part[2 * a.R + kk] = __uint_as_float(v[0]);
-          part[2 * a.R + kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
-        }
-        ++sigcount;
-        if (tid < a.R || h == 0) __threadfence();  // this thread's partials before the arrival count
-        named_bar_sync(kEpiBar, kEpi);
-        if (tid == 0) {
-          // the key norms of this item are published too
-          ok = wait_bar(&s.kpub[slot], qphase, a, 19u);
-          if (ok) pending_old = atom_add_acq_rel(a.sync + 4 + u, 1u);  // resolved at the next loop top
-        }
-        pending_u = u;
+        // the stats warp counts the item once all eight warps have written
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.p1done[slot]);
       } else {  // kP2
-        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 18u))) break;  // statistics copy landed
+        ok = __all_sync(0xffffffffu, wait_bar(&s.qfull[slot], qphase, a, 18u));  // statistics copy landed
         const float* lse = d.ust + ustat_lse();
         const float* kbv = d.ust + ustat_kbar();
         const float ksq = d.ust[ustat_ksq()];
         float s_all = 0.f, mn = INFINITY, mx = -INFINITY, s_de = 0.f, s_c = 0.f, s_raw = 0.f;
-        const uint32_t bmask = (1u << nbuf_log) - 1u;
         for (int t = 0; t < ntiles && ok; ++t) {
           const int i = i0 + t * kTile + kk;
           const bool valid = i < a.N;
           const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
-          if (!(ok = wait_bar(&s.tmem_full[b], tph, a, 14u))) break;
+          if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.tmem_full[b], tph, a, 14u)))) break;
           tc_fence_after();
-          uint32_t rc[RH], stc[8];
+          uint32_t rc[RH];
           tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), rc);
-          if (h == 0) tmem_ld_x8(tl + b * (uint32_t)a.NP + (uint32_t)a.R4, stc);
           tmem_wait_ld();
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
-          const uint32_t par = tcount & 1u;
           ++tcount;
-          float n2 = 0.f;
-          if (h == 0) {
-            // this key's squared norm from the key warps
-            const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
-            if (!(ok = wait_bar(&s.nfull[nb], nph, a, 15u))) break;
-            n2 = s.nbuf[nb][kk];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.nempty[nb]);
-          }
-          ++p2count;
-          // the lse of rows past R is +inf: their terms vanish without a mask
+          const uint32_t ps = pcount % kNB, pph = (pcount / kNB) & 1u;
+          ++pcount;
+          // vote of this half's rows; the lse of rows past R is +inf, so
+          // padding and statistics columns add exactly zero
           float vp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < RH; ++c) vp[c & 3] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -lse[h * RH + c]));
-          s.xch[par][h][kk] = (vp[0] + vp[1]) + (vp[2] + vp[3]);
-          named_bar_sync(kEpiBar, kEpi);
-          if (h == 0 && valid) {
-            const float v = s.xch[par][0][kk] + s.xch[par][1][kk];
-            const float kkb = (__uint_as_float(stc[0]) + __uint_as_float(stc[1])) + __uint_as_float(stc[2]);
-            const float kmu = __uint_as_float(stc[3]) + __uint_as_float(stc[4]);
+          const float vh = (vp[0] + vp[1]) + (vp[2] + vp[3]);
+          if (h == 0) {
+            // hand the first half's vote to the second half
+            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.xempty[ps], pph ^ 1u, a, 24u)))) break;
+            s.xch[ps][kk] = vh;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.xfull[ps]);
+          } else {
+            // the statistics columns (the last eight of the accumulator):
+            // k . kbar in three terms, k . mu in two
+            const float kkb =
+                (__uint_as_float(rc[RH - 8]) + __uint_as_float(rc[RH - 7])) + __uint_as_float(rc[RH - 6]);
+            const float kmu = __uint_as_float(rc[RH - 5]) + __uint_as_float(rc[RH - 4]);
+            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nfull[ps], pph, a, 15u)))) break;
+            const float n2 = s.nbuf[ps][kk];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.nempty[ps]);
             float d2 = fmaf(-2.f, kkb, n2) + ksq;
-            if (d2 < 0.015625f * (n2 + ksq)) {
+            if (valid && d2 < 0.015625f * (n2 + ksq)) {
               // cancellation regime: recompute |k - kbar|^2 from the key row
               const uint4* row = reinterpret_cast<const uint4*>(a.K) + ((size_t)u * a.N + i) * 16;
               float dp[4] = {0.f, 0.f, 0.f, 0.f};
@@ -578,46 +585,56 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const float dEv = sqrtf(fmaxf(d2, 0.f));
             const float cs = kmu * rsqrtf(fmaxf(n2, 1e-24f));
-            s_all += dEv;
-            if (i < a.Tv) {
-              mn = fminf(mn, dEv);
-              mx = fmaxf(mx, dEv);
-              s_de += dEv;
-              s_c += cs;
-              s_raw += v;
-              const size_t o = (size_t)u * a.Tv + i;
-              a.simp[o] = v;
-              a.dE[o] = dEv;
-              a.cosv[o] = cs;
+            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.xfull[ps], pph, a, 25u)))) break;
+            const float v = vh + s.xch[ps][kk];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.xempty[ps]);
+            if (valid) {
+              s_all += dEv;
+              if (i < a.Tv) {
+                mn = fminf(mn, dEv);
+                mx = fmaxf(mx, dEv);
+                s_de += dEv;
+                s_c += cs;
+                s_raw += v;
+                const size_t o = (size_t)u * a.Tv + i;
+                a.simp[o] = v;
+                a.dE[o] = dEv;
+                a.cosv[o] = cs;
+              }
             }
           }
         }
-        if (!ok) break;
-        // the chunk's six partials in one pass: warp butterflies, then the
-        // first warp combines the eight warps in a fixed order
+        // the chunk's six partials: warp butterflies in the second half, then
+        // its first warp combines the four warps in a fixed order
+        if (h == 1) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          s_all += __shfl_xor_sync(0xffffffffu, s_all, o);
-          mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-          s_de += __shfl_xor_sync(0xffffffffu, s_de, o);
-          s_c += __shfl_xor_sync(0xffffffffu, s_c, o);
-          s_raw += __shfl_xor_sync(0xffffffffu, s_raw, o);
+          for (int o = 16; o > 0; o >>= 1) {
+            s_all += __shfl_xor_sync(0xffffffffu, s_all, o);
+            mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            s_de += __shfl_xor_sync(0xffffffffu, s_de, o);
+            s_c += __shfl_xor_sync(0xffffffffu, s_c, o);
+            s_raw += __shfl_xor_sync(0xffffffffu, s_raw, o);
+          }
+          if (lane == 0) {
+            s.red6[e - 4][0] = s_all;
+            s.red6[e - 4][1] = mn;
+            s.red6[e - 4][2] = mx;
+            s.red6[e - 4][3] = s_de;
+            s.red6[e - 4][4] = s_c;
+            s.red6[e - 4][5] = s_raw;
+          }
         }
-        if (lane == 0) {
-          s.red6[e][0] = s_all;
-          s.red6[e][1] = mn;
-          s.red6[e][2] = mx;
-          s.red6[e][3] = s_de;
-          s.red6[e][4] = s_c;
-          s.red6[e][5] = s_raw;
+        if (!epi_sync()) {
+          ok = false;
+          break;
         }
-        named_bar_sync(kEpiBar, kEpi);
         if (tid < 6) {
           float acc = s.red6[0][tid];
 #pragma unroll
-          for (int w8 = 1; w8 < 8; ++w8) {
-            const float x = s.red6[w8][tid];
+          for (int w4 = 1; w4 < 4; ++w4) {
+            const float x = s.red6[w4][tid];
             acc = tid == 1 ? fminf(acc, x) : tid == 2 ? fmaxf(acc, x) : acc + x;
           }
           float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kP2Stride;
@@ -645,7 +662,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
       if (lane == 0) {
         ok = wait_bar(&s.item_empty[slot], qphase ^ 1u, a, 1u);
-        if (ok && it.type == kP2) ok = wait_flag(a.sync + 4 + a.U + it.u, a, 2u);
+        if (ok && it.type == kP2) {
+          ok = wait_flag(a.sync + 4 + a.U + it.u, a, 2u);
+          fence_proxy_async_global();  // the statistics are read next by a bulk copy (async proxy)
+        }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
       if (!ok) break;
@@ -731,6 +751,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
         tc_fence_after();
         const uint32_t qb = smem_u32(s.qbuf[slot]);
+        // The sum MMA of a pass-1 tile needs the key warps' weights; it is
+        // issued after the next tile's logits so that the epilogue is not
+        // held up by the key warps (the last tile of an item flushes it).
+        int pend_stage = -1, pend_t = 0;
+        auto issue_sums = [&](int st, int tt) -> bool {
+          if (!wait_bar(&s.wready[st], (wpar >> st) & 1u, a, 8u)) return false;
+          wpar ^= 1u << st;
+          const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+          if (tt == 0 && !wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u)) return false;
+          tc_fence_after();
+          const uint32_t kt = smem_u32(s.ktile[st]);
+          const uint32_t wb = smem_u32(s.wbuf[st]);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            // A = key tile viewed MN-major (d contiguous): 16 keys per step
+            const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
+            const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
+            mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (tt > 0 || kk > 0) ? 1u : 0u);
+          }
+          mma_commit(&s.empty[st]);
+          return true;
+        };
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.full[stage], sphase, a, 6u))) break;
@@ -745,24 +787,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           mma_commit(&s.tmem_full[b]);
           if (type == kP1) {
-            if (!(ok = wait_bar(&s.wready[stage], (wpar >> stage) & 1u, a, 8u))) break;
-            wpar ^= 1u << stage;
-            const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
-            if (t == 0 && !(ok = wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u))) break;
-            tc_fence_after();
-            const uint32_t wb = smem_u32(s.wbuf[stage]);
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              // A = key tile viewed MN-major (d contiguous): 16 keys per step
-              const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
-              const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
-              mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
+            if (pend_stage >= 0 && !(ok = issue_sums(pend_stage, pend_t))) break;
+            pend_stage = stage;
+            pend_t = t;
+            if (t == ntiles - 1) {
+              if (!(ok = issue_sums(stage, t))) break;
+              pend_stage = -1;
+              mma_commit(&s.sigma_full[sigcount & 1u]);
+              ++sigcount;
             }
-          }
-          mma_commit(&s.empty[stage]);
-          if (type == kP1 && t == ntiles - 1) {
-            mma_commit(&s.sigma_full[sigcount & 1u]);
-            ++sigcount;
+          } else {
+            mma_commit(&s.empty[stage]);
           }
           ++tcount;
           if (++stage == kStages) {
@@ -780,42 +815,74 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+  } else if (warp == 2) {
+    // ------------------------------------------------ stats warp
+    // Counts finished pass-1 items per unit (gpu-scope atomic); the item that
+    // completes a unit folds its chunk partials into the unit statistics and
+    // releases pass 2 of the unit.  Runs beside the epilogue so that neither
+    // the count's round trip nor the fold holds up the tiles.
+    uint32_t p1par = 0u;  // per slot: parity of the next p1done phase
+    for (int seq = 0; ok; ++seq) {
+      const int slot = seq % kIQ;
+      const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+      if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.item_full[slot], qphase, a, 26u)))) break;
+      const ItemDesc& d = s.desc[slot];
+      const int type = d.type, u = d.u;
+      if (type == kExit) break;
+      if (type == kP1) {
+        // the epilogue's partials and the key warps' norms of the item are written
+        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.p1done[slot], (p1par >> slot) & 1u, a, 27u)))) break;
+        p1par ^= 1u << slot;
+        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.kpub[slot], qphase, a, 19u)))) break;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);  // free the slot before the long part
+      if (type == kP1) {
+        // the arrival is a gpu-scope release of everything this CTA wrote for
+        // the item (the mbarrier waits above ordered it before this thread)
+        unsigned old = 0u;
+        if (lane == 0) old = atom_add_acq_rel(a.sync + 4 + u, 1u);
+        old = __shfl_sync(0xffffffffu, old, 0);
+        if (old == (unsigned)(a.nchunks - 1)) {
+          unit_reduce_warp(a, u, lane);
+          __syncwarp();
+          if (lane == 0) st_release(a.sync + 4 + a.U + u, 1u);
+        }
+      }
+    }
   } else if (warp >= kKeyWarp0) {
     // ------------------------------------------------ key warps (12..15)
     const int kk = threadIdx.x - 32 * kKeyWarp0;  // 0..127: this thread's key row of each tile
     int stage = 0;
-    uint32_t sphase = 0, p2count = 0;
+    uint32_t sphase = 0, p2count = 0, sigcount = 0;
     for (int seq = 0; ok; ++seq) {
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-      if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 20u))) break;
+      if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.item_full[slot], qphase, a, 20u)))) break;
       const ItemDesc& d = s.desc[slot];
       const int type = d.type, ntiles = d.ntiles, i0 = d.i0, u = d.u;
       if (type == kExit) break;
       for (int t = 0; t < ntiles && ok; ++t) {
-        if (!(ok = wait_bar(&s.full[stage], sphase, a, 22u))) break;
+        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.full[stage], sphase, a, 22u)))) break;
         const int i = i0 + t * kTile + kk;
         const bool valid = i < a.N;
         if (type == kP1) {
           // squared norm of this thread's key (packed fp32 pairs), kept for
           // pass 2, and the sum weights w = 1/||k|| in three bf16 terms
-          uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+          float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int hb = 0; hb < 2; ++hb) {
             const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
               const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
-              const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-              for (int t2 = 0; t2 < 4; ++t2) {
-                const uint64_t x = pack_f32x2(__uint_as_float(w4[t2] << 16), __uint_as_float(w4[t2] & 0xffff0000u));
-                acc[t2] = ffma2(x, x, acc[t2]);
-              }
+              sq_acc_bf16x2(v.x, acc[0], acc[1]);
+              sq_acc_bf16x2(v.y, acc[2], acc[3]);
+              sq_acc_bf16x2(v.z, acc[4], acc[5]);
+              sq_acc_bf16x2(v.w, acc[6], acc[7]);
             }
           }
-          const float n2 = ((f32x2_lo(acc[0]) + f32x2_hi(acc[0])) + (f32x2_lo(acc[1]) + f32x2_hi(acc[1]))) +
-                           ((f32x2_lo(acc[2]) + f32x2_hi(acc[2])) + (f32x2_lo(acc[3]) + f32x2_hi(acc[3])));
+          const float n2 = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
           if (valid) a.norm2[(size_t)u * a.N + i] = n2;
@@ -840,7 +907,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
           ++p2count;
           const float n2 = valid ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;
-          if (!(ok = wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u))) break;
+          if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u)))) break;
           s.nbuf[nb][kk] = n2;
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.nfull[nb]);
@@ -851,12 +918,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) break;
-      // publish this item's key norms at gpu scope before the epilogue counts
-      // the item as arrived (the fence is cumulative over the warp's stores
-      // ordered before it by __syncwarp)
+      if (type == kP1) {
+        // chunk sums of k and k/||k|| from the sum MMA (TMEM lane = dimension kk)
+        const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+        ++sigcount;
+        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.sigma_full[sb], sph, a, 13u)))) break;
+        tc_fence_after();
+        uint32_t v[4];
+        tmem_ld_x4(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + kSigmaCol + 16u * sb, v);
+        tmem_wait_ld();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.sigma_empty[sb]);
+        float* part = a.p1part + ((size_t)u * a.nchunks + d.chunk) * a.p1_stride;
+        part[kk] = __uint_as_float(v[0]);
+        part[kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
+      }
+      // the item's key norms and sums are written: the stats warp's gpu-scope
+      // arrival (after it has waited for kpub) publishes them
       __syncwarp();
       if (lane == 0) {
-        if (type == kP1) __threadfence();
         mbar_arrive(&s.kpub[slot]);
         mbar_arrive(&s.item_empty[slot]);
       }
@@ -918,7 +999,7 @@ size_t tc_smem_bytes() { return sizeof(Smem<32>) + 1024; }
 int tc_rows_half(int R) {
   const int r4 = (R + 3) & ~3;
   int np = 16;
-  while (np < r4 + 5) np <<= 1;
+  while (np < r4 + 8) np <<= 1;  // window rows, then the statistics rows in the last eight
   return np > kNPMax ? 0 : np / 2;
 }
 
