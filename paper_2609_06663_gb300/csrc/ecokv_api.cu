@@ -77,7 +77,7 @@ static void stage_event(int i, cudaStream_t s) {
 }
 
 // Keys per tensor-core pass item (128 * tiles; ECOKV_TC_TILES overrides the
-// default of 8 tiles for tuning).
+// default of 32 tiles for tuning).
 static int tc_chunk_keys() { return 128 * env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64); }
 
 static int env_int(const char* name, int dflt, int lo, int hi) {
@@ -172,7 +172,11 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.q_rows = p.n_layers * p.h_q * p.window;
   a.tiles_per_chunk = tiles;
   a.nchunks = L.nchunks;
-  a.lag_p2 = env_int("ECOKV_LAG_P2", 10, 1, 64);
+  // pass 2 of unit u is scheduled lag units after its pass 1; a long lag
+  // (all of pass 1 first for up to 64 units) keeps pass-2 items from waiting
+  // on unit statistics still being folded
+  a.lag_p2 = env_int("ECOKV_LAG_P2", 64, 1, 1 << 20);
+  if (a.lag_p2 > L.U) a.lag_p2 = L.U;
   a.total_tickets = (L.U + a.lag_p2) * 2 * a.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;

@@ -2,7 +2,7 @@
 // one launch on sm_103a.
 //
 // Work is a global, ticket-ordered list of items:
-//   P1(u, c)  pass 1 over chunk c (up to 8 tiles of 128 keys) of unit u
+//   P1(u, c)  pass 1 over chunk c (up to 32 tiles of 128 keys) of unit u
 //             (u = (layer, KV head)): window logits (tcgen05 MMA, keys as M,
 //             window rows as N), per-row online-softmax partials, key norms,
 //             and the chunk sums of k and k/||k|| (a second tcgen05 MMA with the
@@ -17,12 +17,13 @@
 //             close to their centroid) the key is recomputed directly from its
 //             row in global memory.
 // Work is a global, ticket-ordered list of items.  Within a schedule step s
-// the list holds P1(s, *) then P2(s - lag_p2, *), so pass 2 of a unit re-reads
-// its keys a few units after pass 1 (from L2 when the keys streamed in
-// between fit), and every item depends only on items with smaller tickets:
-// dispatch is deadlock-free without co-residency.  Pass 2 leaves
-// per-candidate arrays and per-chunk partial sums; finalisation, selection
-// and the gather of the kept rows run in the next launch (finalize_select.cu).
+// the list holds P1(s, *) then P2(s - lag_p2, *): pass 2 of a unit runs lag_p2
+// units after its pass 1 (a short lag re-reads the keys from L2, a long one
+// never waits for unit statistics; the host picks), and every item depends
+// only on items with smaller tickets: dispatch is deadlock-free without
+// co-residency.  Pass 2 leaves per-candidate arrays and per-chunk partial
+// sums; finalisation, selection and the gather of the kept rows run in the
+// next launches (finalize_select.cu).
 //
 // Warp roles (512 threads, one CTA per SM): warp 0 takes tickets, resolves
 // dependencies (bounded spins on gpu-scope flags), loads the window queries

@@ -5,7 +5,7 @@
 
 namespace ecokv {
 
-constexpr int kTcTilesPerChunk = 8;            // default tiles of 128 keys per pass item
+constexpr int kTcTilesPerChunk = 32;           // default tiles of 128 keys per pass item
 constexpr int kTcMinTiles = 2;                 // smallest item the workspace is sized for
 constexpr int kTcChunk = 128 * kTcMinTiles;
 
@@ -13,7 +13,7 @@ struct TcArgs {
   int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
   int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
-  int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1
+  int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1 (<= U)
   int total_tickets;                // (U + lag_p2) * 2 * nchunks
   int p1_stride, ustat_stride;
   float scale_log2;
