@@ -76,11 +76,13 @@ def byte_model(w) -> dict:
 
 def launches_per_call(w) -> int:
     """Kernels one ecokv_evict call launches: the persistent tensor-core
-    streaming kernel (bf16, n >= 128, g*W <= 120) or the two CUDA-core passes,
-    then the finalize/select kernel and the compaction kernel."""
+    streaming kernel (bf16, n >= 128, padded g*W + 8 statistics rows <= 128)
+    or the two CUDA-core passes, then the finalize/select kernel (one thread-
+    block cluster per head, or one CTA per head past 32768 candidates) and the
+    compaction kernel."""
     r = w.group * w.window
-    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 5 <= 128
-    return 3 if tc else 4
+    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 8 <= 128
+    return (1 if tc else 2) + 2
 
 
 # ---------------------------------------------------------------- ranks

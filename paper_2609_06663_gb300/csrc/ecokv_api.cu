@@ -207,6 +207,18 @@ static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const
   return ECOKV_OK;
 }
 
+// Scores (and the top-k) of every unit: one cluster per unit when the unit
+// fits eight CTAs, one CTA per unit otherwise.  Both give the same bits.
+// Scores (and the top-k) of every unit: one cluster per unit when the unit
+// fits eight CTAs, one CTA per unit otherwise.
+static ecokv_status run_finalize(FinalArgs f, int U, bool do_select, cudaStream_t s) {
+  if (!do_select) f.idx = nullptr;
+  const cudaError_t e = launch_finalize_cluster(f, U, false, s);
+  if (e == cudaSuccess) return ECOKV_OK;
+  if (e != cudaErrorNotSupported) return ECOKV_ERR_CUDA;
+  return launch_finalize(f, U, do_select, s) == cudaSuccess ? ECOKV_OK : ECOKV_ERR_CUDA;
+}
+
 }  // namespace ecokv
 
 using namespace ecokv;
@@ -271,7 +283,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
   stage_event(1, s);
-  if (launch_finalize(f, L.U, false, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  if (run_finalize(f, L.U, false, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   stage_event(2, s);
   return ECOKV_OK;
 }
@@ -288,7 +300,11 @@ ecokv_status ecokv_select(const ecokv_params* p, const float* S, int32_t* idx, v
   FinalArgs f = final_args(*p, L, nullptr);
   f.S = const_cast<float*>(S);
   f.idx = idx;
-  if (launch_select(f, L.U, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const cudaError_t e = launch_finalize_cluster(f, L.U, true, s);
+  if (e == cudaSuccess) return ECOKV_OK;
+  if (e != cudaErrorNotSupported) return ECOKV_ERR_CUDA;
+  if (launch_select(f, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   return ECOKV_OK;
 }
 
@@ -334,7 +350,7 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
   stage_event(1, s);
-  if (launch_finalize(f, L.U, true, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  if (run_finalize(f, L.U, true, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   stage_event(2, s);
   if (launch_compact(c, dtype, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   stage_event(3, s);

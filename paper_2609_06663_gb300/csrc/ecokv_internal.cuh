@@ -109,5 +109,9 @@ cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStrea
 // select only, on caller scores f.S
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s);
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
+// One thread-block cluster per unit: scores, and the top-k when f.idx is set
+// (select_only: the top-k of the given scores f.S); cudaErrorNotSupported
+// when the unit is too long for one cluster.
+cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only, cudaStream_t s);
 
 }  // namespace ecokv

@@ -116,7 +116,9 @@ def test_config_c2_two_layers():
     run_and_compare(CONFIGS["c2"], layers=range(5, 7))
 
 
-@pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4)])
+# (65536, 4): more candidates than one thread-block cluster holds, so the
+# finalize runs one CTA per head
+@pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4), (65536, 4)])
 def test_sweep_points(n, window):
     run_and_compare(sweep_workload(n, window))
 
