@@ -28,16 +28,20 @@
 // Warp roles (512 threads, one CTA per SM): warp 0 takes tickets, resolves
 // dependencies (bounded spins on gpu-scope flags), loads the window queries
 // (TMA) and the unit statistics (bulk copy) and issues TMA loads of 32 KB key
-// tiles into a 5-stage ring; warp 1 issues the tcgen05 MMAs into up to four
-// TMEM accumulators (plus two for the sums); warps 12-15 (key warps, one key
-// per thread) compute the key norms and the sum weights of each pass-1 tile
-// as soon as it lands, so that a ring stage is freed without waiting for the
-// softmax, store the norms for pass 2 and hand them to the epilogue there;
-// warps 4-11 are the epilogue (one key per TMEM lane, window rows split in
-// two halves); warps 2-3 idle.  setmaxnreg gives the two epilogue
-// warpgroups 176 registers a thread and the others 80.  Every mbarrier wait and spin
-// is bounded: on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
-// gpu-wide abort flag, drains its own copies and MMAs, frees TMEM and exits.
+// tiles into a 5-stage ring; warp 1 issues the logits MMAs into up to four
+// TMEM accumulators; warp 3 issues the sum MMAs of pass-1 tiles (two more
+// accumulators) as soon as a tile's logits are done and its weights written,
+// and frees the stage; warp 2 counts finished pass-1 items and folds completed
+// units; warps 12-15 (key warps, one key per thread) compute the key norms
+// and the sum weights of each pass-1 tile as soon as it lands, store the norms
+// for pass 2, read the chunk sums, and hand the norms to the epilogue in pass
+// 2; warps 4-11 are the epilogue (one key per TMEM lane, window rows split in
+// two halves).  A stage is held only as long as its own tile needs it: the
+// number of key bytes in flight per SM, not the arithmetic, sets the pace.
+// setmaxnreg gives the two epilogue warpgroups 176 registers a thread and the
+// others 80.  Every mbarrier wait and spin is bounded: on timeout the kernel
+// records ECOKV_ERR_TIMEOUT, raises a gpu-wide abort flag, drains its own
+// copies and MMAs, frees TMEM and exits.
 
 #include <cuda.h>
 #include <stddef.h>
@@ -96,7 +100,8 @@ struct __align__(1024) Smem {
   uint64_t full[kS], empty[kS], wready[kS];
   uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
   uint64_t tmem_full[4], tmem_empty[4];
-  uint64_t sigma_full[2], sigma_empty[2], drain;
+  uint64_t sigma_full[2], sigma_empty[2], drain, drain2;
+  uint64_t lgdone[kS];  // pass-1 tile: its logits MMA is complete (for the sum-MMA issuer)
   float nbuf[kNB][kTile];                        // pass-2 squared key norms, key warps -> epilogue
   uint64_t nfull[kNB], nempty[kNB];
   uint64_t xfull[kNB], xempty[kNB];             // first row half -> second row half, per pass-2 tile
@@ -337,7 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kIQ; ++i) {
       mbar_init(&s.item_full[i], 1);
-      mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps + 1);  // MMA commit + epilogue + key warps + stats warp
+      mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps + 2);  // MMA commit + epilogue + key warps + stats + sum warps
       mbar_init(&s.p1done[i], 8);
       mbar_init(&s.qfull[i], 1);
     }
@@ -358,6 +363,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     s.epi_abort = 0;
     mbar_init(&s.drain, 1);
+    mbar_init(&s.drain2, 1);
+    for (int i = 0; i < kStages; ++i) mbar_init(&s.lgdone[i], 1);
     fence_mbar_init();
   }
   // constant rows of the sum-weight operand: row 0 = 1, rows 4..15 = 0
@@ -738,10 +745,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
       int stage = 0;
-      uint32_t sphase = 0, tcount = 0, sigcount = 0;
-      uint32_t wpar = 0u;  // per stage: parity of the next wready phase (pass-1 tiles only)
+      uint32_t sphase = 0, tcount = 0;
       const uint32_t idesc_l = idesc_bf16(128, a.NP, false, false);
-      const uint32_t idesc_s = idesc_bf16(128, 16, true, false);
       for (int seq = 0; ok; ++seq) {
         const int slot = seq % kIQ;
         const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
@@ -752,28 +757,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
         tc_fence_after();
         const uint32_t qb = smem_u32(s.qbuf[slot]);
-        // The sum MMA of a pass-1 tile needs the key warps' weights; it is
-        // issued after the next tile's logits so that the epilogue is not
-        // held up by the key warps (the last tile of an item flushes it).
-        int pend_stage = -1, pend_t = 0;
-        auto issue_sums = [&](int st, int tt) -> bool {
-          if (!wait_bar(&s.wready[st], (wpar >> st) & 1u, a, 8u)) return false;
-          wpar ^= 1u << st;
-          const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
-          if (tt == 0 && !wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u)) return false;
-          tc_fence_after();
-          const uint32_t kt = smem_u32(s.ktile[st]);
-          const uint32_t wb = smem_u32(s.wbuf[st]);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            // A = key tile viewed MN-major (d contiguous): 16 keys per step
-            const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
-            const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
-            mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (tt > 0 || kk > 0) ? 1u : 0u);
-          }
-          mma_commit(&s.empty[st]);
-          return true;
-        };
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t b = tcount & ((1u << nbuf_log) - 1u), tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = wait_bar(&s.full[stage], sphase, a, 6u))) break;
@@ -787,19 +770,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_bf16(tmem + b * (uint32_t)a.NP, ad, bd, idesc_l, kk > 0 ? 1u : 0u);
           }
           mma_commit(&s.tmem_full[b]);
-          if (type == kP1) {
-            if (pend_stage >= 0 && !(ok = issue_sums(pend_stage, pend_t))) break;
-            pend_stage = stage;
-            pend_t = t;
-            if (t == ntiles - 1) {
-              if (!(ok = issue_sums(stage, t))) break;
-              pend_stage = -1;
-              mma_commit(&s.sigma_full[sigcount & 1u]);
-              ++sigcount;
-            }
-          } else {
-            mma_commit(&s.empty[stage]);
-          }
+          // pass 1: the sum MMA (warp 3) still reads the stage; pass 2: free it
+          mma_commit(type == kP1 ? &s.lgdone[stage] : &s.empty[stage]);
           ++tcount;
           if (++stage == kStages) {
             stage = 0;
@@ -813,6 +785,60 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&s.drain);
         const long long t0 = clock64();
         while (!mbar_try_wait(&s.drain, 0u) && clock64() - t0 < a.timeout_cycles) {
+        }
+      }
+    }
+  } else if (warp == 3) {
+    // ------------------------------------------------ sum-MMA issuer
+    // For each pass-1 tile, once its logits MMA is complete and the key warps
+    // have written the weights: the MMA of the key tile (MN-major view)
+    // against [1, w_hi, w_mid, w_lo] that accumulates the chunk's sums of k
+    // and k/||k||, then the release of the stage.  A thread of its own, so
+    // that neither the logits issuer waits for the key warps nor a stage
+    // waits for the next tile.
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t sigcount = 0, wpar = 0u, lpar = 0u;  // per stage: parity of the next wready / lgdone phase
+      const uint32_t idesc_s = idesc_bf16(128, 16, true, false);
+      for (int seq = 0; ok; ++seq) {
+        const int slot = seq % kIQ;
+        const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
+        if (!(ok = wait_bar(&s.item_full[slot], qphase, a, 28u))) break;
+        const ItemDesc& d = s.desc[slot];
+        const int type = d.type, ntiles = d.ntiles;
+        if (type == kExit) break;
+        mbar_arrive(&s.item_empty[slot]);  // the descriptor is read
+        for (int t = 0; t < ntiles; ++t) {
+          if (type == kP1) {
+            if (!(ok = wait_bar(&s.lgdone[stage], (lpar >> stage) & 1u, a, 29u))) break;
+            lpar ^= 1u << stage;
+            if (!(ok = wait_bar(&s.wready[stage], (wpar >> stage) & 1u, a, 8u))) break;
+            wpar ^= 1u << stage;
+            const uint32_t sb = sigcount & 1u, sph = (sigcount >> 1) & 1u;
+            if (t == 0 && !(ok = wait_bar(&s.sigma_empty[sb], sph ^ 1u, a, 9u))) break;
+            tc_fence_after();
+            const uint32_t kt = smem_u32(s.ktile[stage]);
+            const uint32_t wb = smem_u32(s.wbuf[stage]);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              // A = key tile viewed MN-major (d contiguous): 16 keys per step
+              const uint64_t ad = smem_desc(kt + kk * 2048, kTileBytes / 2, 1024, 2);
+              const uint64_t bd = smem_desc(wb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024, 2);
+              mma_bf16(tmem + kSigmaCol + 16u * sb, ad, bd, idesc_s, (t > 0 || kk > 0) ? 1u : 0u);
+            }
+            mma_commit(&s.empty[stage]);
+            if (t == ntiles - 1) {
+              mma_commit(&s.sigma_full[sb]);
+              ++sigcount;
+            }
+          }
+          if (++stage == kStages) stage = 0;
+        }
+      }
+      if (!ok) {
+        mma_commit(&s.drain2);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(&s.drain2, 0u) && clock64() - t0 < a.timeout_cycles) {
         }
       }
     }
