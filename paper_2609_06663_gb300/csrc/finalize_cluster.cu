@@ -85,6 +85,14 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     // 1. the six pass-2 partials (sum over all N of d_E, min / max / sum of
     //    d_E, sums of cosines and of raw votes over the candidates); meanwhile
     //    the CTA's raw votes with the pooling halo and the edge values
+    // this thread's d_E and cosines, in flight through the scalar phase
+    float e_[kJ], c_[kJ];
+#pragma unroll
+    for (int j = 0; j < kJ; ++j) {
+      const int i = span0 + 32 * j + lane;
+      e_[j] = i < Tv ? __ldg(dEp + i) : 0.f;
+      c_[j] = i < Tv ? __ldg(cvp + i) : 0.f;
+    }
     float v6[6] = {0.f, INFINITY, -INFINITY, 0.f, 0.f, 0.f};
     for (int ch = tid; ch < f.nchunks; ch += kCThreads) {
       const float* p = f.p2part + ((size_t)u * f.nchunks + ch) * kP2Stride;
@@ -117,6 +125,25 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   #pragma unroll
       for (int q = 0; q < 6; ++q) sm.red[warp][q] = v6[q];
     __syncthreads();
+    // pooled importance of the owned candidates (needs no unit scalar)
+  #pragma unroll 4
+    for (int j = 0; j < kJ; ++j) {
+      const int i = span0 + 32 * j + lane;
+      if (i < Tv) {
+        float sp;
+        if (pool_smem) {
+          // the same sum, in the same order, as pooled(); halo entries outside
+          // [0, Tv) hold +0 and leave it unchanged
+          const float* r0 = sm.rawS + (i - lo);
+          float acc = 0.f;
+          for (int o = 0; o <= 2 * hpool; ++o) acc = __fadd_rn(acc, r0[o]);
+          sp = __fdiv_rn(acc, (float)f.pool);
+        } else {
+          sp = pooled(raw, i, Tv, f.pool);
+        }
+        sm.buf[i - lo] = __float_as_uint(sp);
+      }
+    }
     if (tid == 0) {
       float s_all = sm.red[0][0], mnE = sm.red[0][1], mxE = sm.red[0][2];
       float s_de = sm.red[0][3], s_c = sm.red[0][4], s_raw = sm.red[0][5];
@@ -148,27 +175,15 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     __syncthreads();
     const float lamf = sm.sc[0], mnE = sm.sc[1], denE = sm.sc[2];
 
-    // 2. S_div (Eq. 2, 3) and pooled importance of the owned candidates
+    // 2. S_div (Eq. 2, 3) of the owned candidates and its extrema
     float mnD = INFINITY, mxD = -INFINITY;
-  #pragma unroll 8
+  #pragma unroll
     for (int j = 0; j < kJ; ++j) {
       const int i = span0 + 32 * j + lane;
       if (i < Tv) {
-        const float sd = sdiv_of(__ldg(dEp + i), __ldg(cvp + i), mnE, denE, f.alpha, mix);
+        const float sd = sdiv_of(e_[j], c_[j], mnE, denE, f.alpha, mix);
         mnD = fminf(mnD, sd);
         mxD = fmaxf(mxD, sd);
-        float sp;
-        if (pool_smem) {
-          // the same sum, in the same order, as pooled(); halo entries outside
-          // [0, Tv) hold +0 and leave it unchanged
-          const float* r0 = sm.rawS + (i - lo);
-          float acc = 0.f;
-          for (int o = 0; o <= 2 * hpool; ++o) acc = __fadd_rn(acc, r0[o]);
-          sp = __fdiv_rn(acc, (float)f.pool);
-        } else {
-          sp = pooled(raw, i, Tv, f.pool);
-        }
-        sm.buf[i - lo] = __float_as_uint(sp);
       }
     }
   #pragma unroll
@@ -232,11 +247,11 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     //    importance in buf
     float* Sg = f.S ? f.S + (size_t)u * Tv : nullptr;
     float* dbg = f.dbg ? f.dbg + (size_t)u * 5 * Tv : nullptr;
-  #pragma unroll 8
+  #pragma unroll
     for (int j = 0; j < kJ; ++j) {
       const int i = span0 + 32 * j + lane;
       if (i < Tv) {
-        const float e = __ldg(dEp + i), c = __ldg(cvp + i);
+        const float e = e_[j], c = c_[j];
         const float sd = sdiv_of(e, c, mnE, denE, f.alpha, mix);
         const float sbar = __fdiv_rn(__fsub_rn(sd, mnD2), denD);
         const float sp = __uint_as_float(sm.buf[i - lo]);
