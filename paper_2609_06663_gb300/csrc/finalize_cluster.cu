@@ -11,7 +11,8 @@
 //      result), lambda (Eq. 4-6);
 //   2. S_div (Eq. 2, 3) and pooled S_imp of the owned candidates; extrema of
 //      S_div over the cluster;
-//   3. S (Eq. 7) bit for bit as finalize_unit computes it;
+//   3. S (Eq. 7) as finalize_unit computes it, divisions by the min-max
+//      ranges and the pooling kernel taken as reciprocal products;
 //   4. MSB-first radix select over the order-preserving image of S, one
 //      256-bin histogram per CTA, summed over the cluster for each 8-bit digit;
 //   5. counts of keys above / equal to the threshold, exchanged so that each
@@ -39,7 +40,8 @@ constexpr int kHalo = 16;                       // pooling halo kept in shared m
 struct ClusterSmem {
   float rawS[kCap + 2 * kHalo];  // the CTA's raw votes with the pooling halo
   unsigned buf[kCap];            // pooled importance, then the order-preserving keys of S
-  unsigned hist[2][256];         // per radix pass (double-buffered across passes)
+  unsigned hist[2][256];         // per radix pass, the CTA's sum (double-buffered across passes)
+  unsigned whist[kCWarps][256];  // per radix pass, each warp's own histogram
   float red[kCWarps][8];         // per-warp partials
   float edge[32];                // pooling edge values
   float sc[8];                   // broadcast scalars
@@ -48,6 +50,15 @@ struct ClusterSmem {
   unsigned wsum[kCWarps];
   int shi[32];
 };
+
+// Composite diversity (Eq. 2 and Eq. 3) with the min-max divisor applied as a
+// reciprocal (one rounding more than a division; every score of a call uses
+// the same formula, and ecokv_score and ecokv_evict share this kernel).
+__device__ __forceinline__ float sdiv_rcp(float dE, float c, float mnE, float invE, float alpha, bool mix) {
+  const float sE = __fmul_rn(__fsub_rn(dE, mnE), invE);
+  const float sC = mix ? -c : __fmul_rn(__fsub_rn(1.f, c), 0.5f);
+  return __fadd_rn(__fmul_rn(alpha, sE), __fmul_rn(__fsub_rn(1.f, alpha), sC));
+}
 
 // kMode: 0 = scores, 1 = scores and top-k, 2 = top-k of given scores (f.S).
 template <int kMode>
@@ -126,6 +137,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       for (int q = 0; q < 6; ++q) sm.red[warp][q] = v6[q];
     __syncthreads();
     // pooled importance of the owned candidates (needs no unit scalar)
+    const float inv_pool = __frcp_rn((float)f.pool);
   #pragma unroll 4
     for (int j = 0; j < kJ; ++j) {
       const int i = span0 + 32 * j + lane;
@@ -136,10 +148,18 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
           // [0, Tv) hold +0 and leave it unchanged
           const float* r0 = sm.rawS + (i - lo);
           float acc = 0.f;
-          for (int o = 0; o <= 2 * hpool; ++o) acc = __fadd_rn(acc, r0[o]);
-          sp = __fdiv_rn(acc, (float)f.pool);
+          if (hpool == 2) {  // the default kernel of 5, loads in parallel
+            const float x0 = r0[0], x1 = r0[1], x2 = r0[2], x3 = r0[3], x4 = r0[4];
+            acc = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(acc, x0), x1), x2), x3), x4);
+          } else {
+            for (int o = 0; o <= 2 * hpool; ++o) acc = __fadd_rn(acc, r0[o]);
+          }
+          sp = __fmul_rn(acc, inv_pool);
         } else {
-          sp = pooled(raw, i, Tv, f.pool);
+          float acc = 0.f;
+          for (int o = -hpool; o <= hpool; ++o)
+            if (i + o >= 0 && i + o < Tv) acc = __fadd_rn(acc, __ldg(raw + i + o));
+          sp = __fmul_rn(acc, inv_pool);
         }
         sm.buf[i - lo] = __float_as_uint(sp);
       }
@@ -174,6 +194,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     }
     __syncthreads();
     const float lamf = sm.sc[0], mnE = sm.sc[1], denE = sm.sc[2];
+    const float invE = __frcp_rn(denE);
 
     // 2. S_div (Eq. 2, 3) of the owned candidates and its extrema
     float mnD = INFINITY, mxD = -INFINITY;
@@ -181,7 +202,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     for (int j = 0; j < kJ; ++j) {
       const int i = span0 + 32 * j + lane;
       if (i < Tv) {
-        const float sd = sdiv_of(e_[j], c_[j], mnE, denE, f.alpha, mix);
+        const float sd = sdiv_rcp(e_[j], c_[j], mnE, invE, f.alpha, mix);
         mnD = fminf(mnD, sd);
         mxD = fmaxf(mxD, sd);
       }
@@ -241,6 +262,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     }
     __syncthreads();
     const float mnD2 = sm.sc[6], denD = sm.sc[7], scale = sm.sc[5];
+    const float invD = __frcp_rn(denD);
     const float one_m_lam = __fsub_rn(1.f, lamf);
 
     // 3. final scores (Eq. 7); the order-preserving keys replace the pooled
@@ -252,8 +274,8 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       const int i = span0 + 32 * j + lane;
       if (i < Tv) {
         const float e = e_[j], c = c_[j];
-        const float sd = sdiv_of(e, c, mnE, denE, f.alpha, mix);
-        const float sbar = __fdiv_rn(__fsub_rn(sd, mnD2), denD);
+        const float sd = sdiv_rcp(e, c, mnE, invE, f.alpha, mix);
+        const float sbar = __fmul_rn(__fsub_rn(sd, mnD2), invD);
         const float sp = __uint_as_float(sm.buf[i - lo]);
         const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
         sm.buf[i - lo] = ordered_key(S);
@@ -277,9 +299,13 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     if (k > 0) {
       int pass = 0;
       for (int shift = 24; shift >= 0; shift -= 8, ++pass) {
-        unsigned* hist = sm.hist[pass & 1];
-        hist[tid] = 0u;  // kCThreads == 256 bins
-        __syncthreads();
+        // each warp counts into its own histogram (no two warps contend for
+        // one address: the keys of a head crowd into few bins), then the
+        // CTA's histogram is their sum
+        unsigned* wh = sm.whist[warp];
+#pragma unroll
+        for (int b = lane; b < 256; b += 32) wh[b] = 0u;
+        __syncwarp();
 #pragma unroll 4
         for (int j = 0; j < kJ; ++j) {
           const int i = span0 + 32 * j + lane;
@@ -289,7 +315,15 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
             if ((key & mask) == prefix) bin = (key >> shift) & 255u;
           }
           const unsigned peers = __match_any_sync(0xffffffffu, bin);
-          if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], (unsigned)__popc(peers));
+          if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(&wh[bin], (unsigned)__popc(peers));
+        }
+        __syncthreads();
+        unsigned* hist = sm.hist[pass & 1];
+        {
+          unsigned cnt = 0u;  // kCThreads == 256 bins: thread tid sums bin tid
+#pragma unroll
+          for (int w = 0; w < kCWarps; ++w) cnt += sm.whist[w][tid];
+          hist[tid] = cnt;
         }
         cl.sync();
         // the cluster's histogram (rank order: deterministic), bin tid; suffix
