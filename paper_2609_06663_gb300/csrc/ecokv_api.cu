@@ -76,9 +76,19 @@ static void stage_event(int i, cudaStream_t s) {
   if (g_stage_ev[i] != nullptr) cudaEventRecord(g_stage_ev[i], s);
 }
 
-// Keys per tensor-core pass item (128 * tiles; ECOKV_TC_TILES overrides the
-// default of 32 tiles for tuning).
-static int tc_chunk_keys() { return 128 * env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64); }
+// Tiles of 128 keys per tensor-core pass item: the largest power of two up
+// to 64 that still leaves at least two items per SM (152 SMs) in each
+// pass, so that the persistent grid stays busy to its end while the per-item
+// costs (statistics, partial sums, scheduling) stay few.  ECOKV_TC_TILES
+// overrides it for tuning.
+static int tc_tiles(const ecokv_params& p) {
+  constexpr long long kItemsWanted = 2LL * 152;
+  int t = kTcMaxTiles;
+  const long long U = (long long)p.n_layers * p.h_kv;
+  while (t > kTcMinTiles && U * ((p.n + 128LL * t - 1) / (128LL * t)) < kItemsWanted) t >>= 1;
+  return env_int("ECOKV_TC_TILES", t, kTcMinTiles, kTcMaxTiles);
+}
+static int tc_chunk_keys(const ecokv_params& p) { return 128 * tc_tiles(p); }
 
 static int env_int(const char* name, int dflt, int lo, int hi) {
   const char* v = getenv(name);
@@ -155,7 +165,7 @@ static CompactArgs compact_args(const ecokv_params& p, const void* K, const void
 // Both streaming passes on the tensor cores in one launch (after clearing
 // the per-call counters).
 static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
-  const int tiles = env_int("ECOKV_TC_TILES", kTcTilesPerChunk, kTcMinTiles, 64);
+  const int tiles = tc_tiles(p);
   const Layout L = make_layout(p, 128 * tiles);
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   TcArgs a{};
@@ -172,12 +182,13 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.q_rows = p.n_layers * p.h_q * p.window;
   a.tiles_per_chunk = tiles;
   a.nchunks = L.nchunks;
-  // pass 2 of unit u is scheduled lag units after its pass 1; a long lag
-  // (all of pass 1 first for up to 64 units) keeps pass-2 items from waiting
-  // on unit statistics still being folded
-  a.lag_p2 = env_int("ECOKV_LAG_P2", 64, 1, 1 << 20);
+  // pass 2 of unit u is scheduled lag units after its pass 1.  By default all
+  // of pass 1 runs first: pass-2 items then never wait for unit statistics,
+  // and the keys of a unit are gone from L2 by its pass 2 at any lag longer
+  // than the items in flight, so nothing is lost (ECOKV_LAG_P2 for tuning)
+  a.lag_p2 = env_int("ECOKV_LAG_P2", 1 << 20, 1, 1 << 20);
   if (a.lag_p2 > L.U) a.lag_p2 = L.U;
-  a.total_tickets = (L.U + a.lag_p2) * 2 * a.nchunks;
+  a.total_tickets = 2 * L.U * a.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
@@ -274,7 +285,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys() : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.lambda = lambda;
@@ -339,7 +350,7 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys() : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);

@@ -148,20 +148,36 @@ struct Item {
   bool valid;
 };
 
-// Item of a ticket: step s = ticket / (2 * nchunks) holds the P1 items of unit
-// s and then the P2 items of unit s - lag_p2 (invalid outside [0, U)).
+// Item of a ticket.  Schedule step s holds the P1 items of unit s and then
+// the P2 items of unit s - lag_p2; steps are numbered so that no ticket falls
+// outside [0, U): the first lag_p2 steps hold P1 items only, the last lag_p2
+// steps P2 items only, 2 * U * nchunks tickets in all.  lag_p2 = U runs all of
+// pass 1 before any of pass 2.
 __device__ Item decode(int ticket, const TcArgs& a) {
   Item it{kExit, 0, 0, 0, true};
   if (ticket >= a.total_tickets) return it;
-  const int s = ticket / (2 * a.nchunks), slot = ticket - s * 2 * a.nchunks;
-  if (slot < a.nchunks) {
+  const int nc = a.nchunks, L = a.lag_p2;
+  const int head = L * nc, body = (a.U - L) * 2 * nc;
+  if (ticket < head) {
     it.type = kP1;
-    it.u = s;
-    it.chunk = slot;
+    it.u = ticket / nc;
+    it.chunk = ticket - it.u * nc;
+  } else if (ticket < head + body) {
+    const int rel = ticket - head, st = rel / (2 * nc), slot = rel - st * 2 * nc;
+    if (slot < nc) {
+      it.type = kP1;
+      it.u = L + st;
+      it.chunk = slot;
+    } else {
+      it.type = kP2;
+      it.u = st;
+      it.chunk = slot - nc;
+    }
   } else {
+    const int rel = ticket - head - body, v = rel / nc;
     it.type = kP2;
-    it.u = s - a.lag_p2;
-    it.chunk = slot - a.nchunks;
+    it.u = a.U - L + v;
+    it.chunk = rel - v * nc;
   }
   it.valid = it.u >= 0 && it.u < a.U;
   return it;

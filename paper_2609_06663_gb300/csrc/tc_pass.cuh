@@ -5,7 +5,7 @@
 
 namespace ecokv {
 
-constexpr int kTcTilesPerChunk = 32;           // default tiles of 128 keys per pass item
+constexpr int kTcMaxTiles = 64;                // largest item: 64 tiles of 128 keys
 constexpr int kTcMinTiles = 2;                 // smallest item the workspace is sized for
 constexpr int kTcChunk = 128 * kTcMinTiles;
 
@@ -14,7 +14,7 @@ struct TcArgs {
   int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
   int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1 (<= U)
-  int total_tickets;                // (U + lag_p2) * 2 * nchunks
+  int total_tickets;                // 2 * U * nchunks
   int p1_stride, ustat_stride;
   float scale_log2;
   long long timeout_cycles;
