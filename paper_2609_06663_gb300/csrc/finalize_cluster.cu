@@ -1,12 +1,21 @@
 // Finalisation and selection of one (layer, KV head) unit by a thread-block
-// cluster of C CTAs (C <= 8): the arithmetic of finalize_unit / select_unit
+// cluster of C CTAs: the arithmetic of finalize_unit / select_unit
 // (finalize_select.cuh), spread over the cluster so that every SM takes part,
 // with the cluster-wide reductions done through distributed shared memory.
 //
+// Two shapes: 16 candidates a thread and up to 8 CTAs (units up to 32768
+// candidates, used up to 16384), or 32 candidates a thread and up to 4 CTAs
+// (units of 16385 to 32768): at four CTAs per SM the GPU holds about 74
+// clusters of 8 but 148 of 4, so the long units of a prefill (e.g. 28 layers
+// x 4 KV heads of 32k tokens) run in one wave instead of one and a half.
+//
 // CTA rank r of the cluster owns candidates [r * cap, (r + 1) * cap) of the
-// unit (cap = 8 warps x 32 lanes x kJ); warp w of it owns a contiguous span of
-// 32 * kJ of those, lane l position span0 + 32 j + l for j < kJ, kept in
-// registers from the first load to the emitted index.  Steps:
+// unit (cap = 256 threads x kJ); thread t of it owns the kJ consecutive
+// candidates from r * cap + kJ * t and keeps their pooled importance, then
+// the keys of their scores, in registers.  The raw votes of the CTA (with the
+// pooling halo) are staged in shared memory with one pad word after every 32,
+// so that the 32 lanes of a warp, kJ positions apart, read distinct banks.
+// Steps:
 //   1. unit scalars from the pass-2 partials (every CTA, same inputs, same
 //      result), lambda (Eq. 4-6);
 //   2. S_div (Eq. 2, 3) and pooled S_imp of the owned candidates; extrema of
@@ -15,11 +24,15 @@
 //      ranges and the pooling kernel taken as reciprocal products;
 //   4. MSB-first radix select over the order-preserving image of S, one
 //      256-bin histogram per CTA, summed over the cluster for each 8-bit digit;
-//   5. counts of keys above / equal to the threshold, exchanged so that each
-//      CTA knows how many kept candidates precede it (ties to the lower
-//      position), then its kept positions in ascending order (the last CTA
-//      adds the window).  The gather of the kept rows is its own launch.
+//   5. counts of keys above / equal to the threshold, scanned over the
+//      threads and exchanged between the CTAs, so that each thread knows how
+//      many kept candidates precede its own (ties to the lower position);
+//      then its kept positions in ascending order (the last CTA adds the
+//      window).  The gather of the kept rows is its own launch.
 // Cluster barriers are reached by every CTA on every path (no early exit).
+// Every exchange between CTAs is a store into the peers' shared memory
+// (each CTA keeps every rank's contribution) followed by a cluster barrier,
+// so no CTA waits on a remote load.
 
 #include <cooperative_groups.h>
 
@@ -32,23 +45,36 @@ namespace {
 
 constexpr int kCThreads = 256;
 constexpr int kCWarps = kCThreads / 32;
-constexpr int kJ = 16;                          // candidates a thread owns
-constexpr int kCap = kCThreads * kJ;            // candidates a CTA owns
-constexpr int kMaxCluster = 8;
-constexpr int kHalo = 16;                       // pooling halo kept in shared memory (kernel <= 33)
+constexpr int kHalo = 16;  // pooling halo kept in shared memory (kernel <= 33)
 
+template <int kJ>
+struct Shape {
+  static constexpr int kCap = kCThreads * kJ;          // candidates a CTA owns
+  static constexpr int kMaxCluster = kJ == 16 ? 8 : 4;  // CTAs a unit may take
+  static constexpr int kQ = kCap + 2 * kHalo;          // staged raw votes
+};
+
+// Padded shared-memory index of staged position q.
+__device__ __forceinline__ int pad_idx(int q) { return q + (q >> 5); }
+
+template <int kJ>
 struct ClusterSmem {
-  float rawS[kCap + 2 * kHalo];  // the CTA's raw votes with the pooling halo
-  unsigned buf[kCap];            // pooled importance, then the order-preserving keys of S
-  unsigned hist[2][256];         // per radix pass, the CTA's sum (double-buffered across passes)
+  // raw vote of candidate lo - kHalo + q at raw[pad_idx(q)]
+  float raw[Shape<kJ>::kQ + Shape<kJ>::kQ / 32 + 1];
   unsigned whist[kCWarps][256];  // per radix pass, each warp's own histogram
-  float red[kCWarps][8];         // per-warp partials
-  float edge[32];                // pooling edge values
-  float sc[8];                   // broadcast scalars
-  float ext[2];                  // this CTA's min / max of S_div
-  int cnt[2];                    // this CTA's keys above / equal to the threshold
+  // Written by the peers (distributed shared memory stores): per radix pass
+  // the histogram of every rank (double-buffered across passes), the S_div
+  // extrema and the counts above / equal to the threshold of every rank.
+  unsigned hall[2][Shape<kJ>::kMaxCluster][256];
+  float ext_all[Shape<kJ>::kMaxCluster][2];
+  int cnt_all[Shape<kJ>::kMaxCluster][2];
+  float red[kCWarps][8];  // per-warp partials
+  float edge[32];         // pooling edge values
+  float sc[8];            // broadcast scalars
+  double dsc[2];          // sums behind the means of S_imp and of S_div
   unsigned wsum[kCWarps];
-  int shi[32];
+  int wscan[kCWarps][2];  // per-warp counts above / equal to the threshold
+  int shi[4];
 };
 
 // Composite diversity (Eq. 2 and Eq. 3) with the min-max divisor applied as a
@@ -60,20 +86,34 @@ __device__ __forceinline__ float sdiv_rcp(float dE, float c, float mnE, float in
   return __fadd_rn(__fmul_rn(alpha, sE), __fmul_rn(__fsub_rn(1.f, alpha), sC));
 }
 
+// Store v into the same object of every CTA of the cluster (its own included).
+template <int kMaxC, typename T>
+__device__ __forceinline__ void push_all(cg::cluster_group& cl, T* obj, T v, int C) {
+#pragma unroll
+  for (int r = 0; r < kMaxC; ++r)
+    if (r < C) *cl.map_shared_rank(obj, r) = v;
+}
+
 // kMode: 0 = scores, 1 = scores and top-k, 2 = top-k of given scores (f.S).
-template <int kMode>
+template <int kMode, int kJ>
 __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArgs f) {
   constexpr bool kSelect = kMode != 0;
+  constexpr int kCap = Shape<kJ>::kCap, kMaxC = Shape<kJ>::kMaxCluster;
   extern __shared__ __align__(16) uint8_t fc_smem[];
-  ClusterSmem& sm = *reinterpret_cast<ClusterSmem*>(fc_smem);
+  ClusterSmem<kJ>& sm = *reinterpret_cast<ClusterSmem<kJ>*>(fc_smem);
   cg::cluster_group cl = cg::this_cluster();
+  // The peers must have started before the first store into their shared
+  // memory: this arrival is waited for just before it.
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
   const int C = (int)cl.num_blocks();
   const int rank = (int)cl.block_rank();
   const int u = blockIdx.x / C;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int Tv = f.Tv;
-  const int lo = rank * kCap;                      // first candidate of this CTA
-  const int span0 = lo + warp * 32 * kJ;           // first candidate of this warp
+  const int lo = rank * kCap;       // first candidate of this CTA
+  const int c0 = lo + kJ * tid;     // first candidate of this thread
+  const int q0 = kJ * tid + kHalo;  // staged position of candidate c0
+  const int nv = max(0, min(kJ, Tv - c0));  // of this thread's candidates, those below Tv
   const bool keep_all = f.budget >= f.N;
   const int k = keep_all ? 0 : f.budget - f.W;
   const bool mix = (f.flags & ECOKV_FLAG_SC_MIXKV_SIGN) != 0;
@@ -81,29 +121,29 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   const bool pool_smem = hpool <= kHalo;
   const float* us = f.ustat + (size_t)u * f.ustat_stride;
   const float* raw = f.simp + (size_t)u * Tv;
-  const float* dEp = f.dE + (size_t)u * Tv;
-  const float* cvp = f.cosv + (size_t)u * Tv;
+
+  // pooled importance (as float bits), then the order-preserving keys of S
+  unsigned key[kJ];
 
   if (kMode == 2) {
-    // scores given (absent when nothing is to be chosen): their
-    // order-preserving keys
-    if (k > 0)
+    // scores given (absent when nothing is to be chosen): staged in
+    // coalesced order, then each thread's keys
+    if (k > 0) {
+      const float* Su = f.S + (size_t)u * Tv;
+#pragma unroll 8
       for (int j = 0; j < kJ; ++j) {
-        const int i = span0 + 32 * j + lane;
-        if (i < Tv) sm.buf[i - lo] = ordered_key(__ldg(f.S + (size_t)u * Tv + i));
+        const int i = lo + kCThreads * j + tid;
+        if (i < Tv) sm.raw[pad_idx(i - lo + kHalo)] = __ldg(Su + i);
       }
+      __syncthreads();
+#pragma unroll
+      for (int c = 0; c < kJ; ++c) key[c] = ordered_key(sm.raw[pad_idx(q0 + c)]);
+    }
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
   } else {
     // 1. the six pass-2 partials (sum over all N of d_E, min / max / sum of
     //    d_E, sums of cosines and of raw votes over the candidates); meanwhile
     //    the CTA's raw votes with the pooling halo and the edge values
-    // this thread's d_E and cosines, in flight through the scalar phase
-    float e_[kJ], c_[kJ];
-#pragma unroll
-    for (int j = 0; j < kJ; ++j) {
-      const int i = span0 + 32 * j + lane;
-      e_[j] = i < Tv ? __ldg(dEp + i) : 0.f;
-      c_[j] = i < Tv ? __ldg(cvp + i) : 0.f;
-    }
     float v6[6] = {0.f, INFINITY, -INFINITY, 0.f, 0.f, 0.f};
     for (int ch = tid; ch < f.nchunks; ch += kCThreads) {
       const float* p = f.p2part + ((size_t)u * f.nchunks + ch) * kP2Stride;
@@ -115,9 +155,9 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       v6[5] += __ldg(p + P2_SUM_RAW);
     }
     if (pool_smem)
-      for (int q = tid; q < kCap + 2 * hpool; q += kCThreads) {
-        const int j = lo - hpool + q;
-        sm.rawS[q] = (j >= 0 && j < Tv) ? __ldg(raw + j) : 0.f;
+      for (int q = kHalo - hpool + tid; q < kHalo + kCap + hpool; q += kCThreads) {
+        const int j = lo - kHalo + q;
+        sm.raw[pad_idx(q)] = (j >= 0 && j < Tv) ? __ldg(raw + j) : 0.f;
       }
     if (warp == 1 && lane < 2 * hpool && pool_smem) {
       const int j = lane < hpool ? lane : Tv - 2 * hpool + lane;
@@ -136,32 +176,38 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   #pragma unroll
       for (int q = 0; q < 6; ++q) sm.red[warp][q] = v6[q];
     __syncthreads();
-    // pooled importance of the owned candidates (needs no unit scalar)
-    const float inv_pool = __frcp_rn((float)f.pool);
-  #pragma unroll 4
-    for (int j = 0; j < kJ; ++j) {
-      const int i = span0 + 32 * j + lane;
-      if (i < Tv) {
-        float sp;
-        if (pool_smem) {
-          // the same sum, in the same order, as pooled(); halo entries outside
-          // [0, Tv) hold +0 and leave it unchanged
-          const float* r0 = sm.rawS + (i - lo);
-          float acc = 0.f;
-          if (hpool == 2) {  // the default kernel of 5, loads in parallel
-            const float x0 = r0[0], x1 = r0[1], x2 = r0[2], x3 = r0[3], x4 = r0[4];
-            acc = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(acc, x0), x1), x2), x3), x4);
-          } else {
-            for (int o = 0; o <= 2 * hpool; ++o) acc = __fadd_rn(acc, r0[o]);
-          }
-          sp = __fmul_rn(acc, inv_pool);
-        } else {
-          float acc = 0.f;
-          for (int o = -hpool; o <= hpool; ++o)
-            if (i + o >= 0 && i + o < Tv) acc = __fadd_rn(acc, __ldg(raw + i + o));
-          sp = __fmul_rn(acc, inv_pool);
+
+    // pooled importance of the owned candidates (needs no unit scalar): the
+    // same sum, in the same order, as pooled(); halo entries outside [0, Tv)
+    // hold +0 and leave it unchanged
+    {
+      const float inv_pool = __frcp_rn((float)f.pool);
+      if (pool_smem && hpool == 2) {
+        // the default kernel of 5: each staged vote read once
+        float x[kJ + 4];
+#pragma unroll
+        for (int s = 0; s < kJ + 4; ++s) x[s] = sm.raw[pad_idx(q0 - 2 + s)];
+#pragma unroll
+        for (int c = 0; c < kJ; ++c) {
+          const float acc = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(0.f, x[c]), x[c + 1]), x[c + 2]),
+                                                x[c + 3]), x[c + 4]);
+          key[c] = __float_as_uint(c < nv ? __fmul_rn(acc, inv_pool) : 0.f);
         }
-        sm.buf[i - lo] = __float_as_uint(sp);
+      } else {
+#pragma unroll
+        for (int c = 0; c < kJ; ++c) {
+          float acc = 0.f;
+          if (c < nv) {
+            if (pool_smem) {
+              for (int o = -hpool; o <= hpool; ++o) acc = __fadd_rn(acc, sm.raw[pad_idx(q0 + c + o)]);
+            } else {
+              const int i = c0 + c;
+              for (int o = -hpool; o <= hpool; ++o)
+                if (i + o >= 0 && i + o < Tv) acc = __fadd_rn(acc, __ldg(raw + i + o));
+            }
+          }
+          key[c] = __float_as_uint(__fmul_rn(acc, inv_pool));
+        }
       }
     }
     if (tid == 0) {
@@ -175,36 +221,71 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         s_c += sm.red[w][4];
         s_raw += sm.red[w][5];
       }
-      // per-head redundancy and lambda (Eq. 4-6), a few scalar ops in double
-      const double N = (double)f.N;
-      const double D_E = (double)s_all / N;
-      const double tau = f.tau > 0.f ? (double)f.tau : sqrt((double)kD);
-      const double r_E = 2.0 - 2.0 / (1.0 + exp(-D_E / tau));
-      const double mu_sq = (double)__ldg(us + ustat_musq());
-      const double r_C = f.N == 1 ? 1.0 : (N * mu_sq - 1.0) / (N - 1.0);
-      double lam = (double)f.beta * r_E + (1.0 - (double)f.beta) * r_C;
-      if (f.flags & ECOKV_FLAG_LAMBDA_OVERRIDE) lam = (double)f.lambda_override;
-      sm.sc[0] = (float)lam;
+      sm.sc[0] = s_all;
       sm.sc[1] = mnE;
       sm.sc[2] = __fadd_rn(__fsub_rn(mxE, mnE), f.eps);
       sm.sc[3] = s_de;
       sm.sc[4] = s_c;
       sm.sc[5] = s_raw;
-      if (f.lambda != nullptr && rank == 0) f.lambda[u] = (float)lam;
     }
+    // (this barrier also ends every thread's reads of the staged raw votes)
     __syncthreads();
-    const float lamf = sm.sc[0], mnE = sm.sc[1], denE = sm.sc[2];
+    const float mnE = sm.sc[1], denE = sm.sc[2];
     const float invE = __frcp_rn(denE);
 
-    // 2. S_div (Eq. 2, 3) of the owned candidates and its extrema
+    if (tid == 32) {
+      // off the critical path, while the other threads compute S_div:
+      // per-head redundancy and lambda (Eq. 4-6) in single precision (lambda
+      // weighs two terms of order one: its rounding stays at the level of the
+      // scores' own), and the parts of the means that need no cluster extremum
+      const float D_E = __fdiv_rn(sm.sc[0], (float)f.N);
+      const float tau = f.tau > 0.f ? f.tau : sqrtf((float)kD);
+      const float r_E = 2.f - 2.f / (1.f + expf(-D_E / tau));
+      const float mu_sq = __ldg(us + ustat_musq());
+      const float r_C = f.N == 1 ? 1.f : ((float)f.N * mu_sq - 1.f) / (float)(f.N - 1);
+      float lam = f.beta * r_E + (1.f - f.beta) * r_C;
+      if (f.flags & ECOKV_FLAG_LAMBDA_OVERRIDE) lam = f.lambda_override;
+      if (f.lambda != nullptr && rank == 0) f.lambda[u] = lam;
+      sm.sc[0] = lam;
+      // means, in double and scaled by Tv: sum_i S_imp(i) = (1/kp) sum_j
+      // raw(j) cnt(j), where cnt(j) = kp except within kp/2 of either end;
+      // mean(Sbar) is affine in the means of d_E and of the cosine (as
+      // finalize_unit)
+      const int h = hpool;
+      double edge = 0.0;
+      if (pool_smem) {
+        // sm.edge[l] = raw[l] for l < h, raw[Tv - 2h + l] for h <= l < 2h
+        for (int j = 0; j < Tv && j < h; ++j) edge += (double)sm.edge[j] * (double)(h - j);
+        for (int j = (Tv - h > 0 ? Tv - h : 0); j < Tv; ++j)
+          edge += (double)sm.edge[j - Tv + 2 * h] * (double)(h - (Tv - 1 - j));
+      } else {
+        for (int j = 0; j < Tv && j < h; ++j) edge += (double)__ldg(raw + j) * (double)(h - j);
+        for (int j = (Tv - h > 0 ? Tv - h : 0); j < Tv; ++j) edge += (double)__ldg(raw + j) * (double)(h - (Tv - 1 - j));
+      }
+      const double T = (double)Tv;
+      const double sum_sE = ((double)sm.sc[3] - (double)mnE * T) / (double)denE;
+      const double sum_cs = (double)sm.sc[4];
+      const double sum_sC = mix ? -sum_cs : (T - sum_cs) * 0.5;
+      sm.dsc[0] = (double)f.pool * (double)sm.sc[5] - edge;                      // kp * Tv * mean(S_imp)
+      sm.dsc[1] = (double)f.alpha * sum_sE + (1.0 - (double)f.alpha) * sum_sC;  // Tv * mean(S_div)
+    }
+
+    // 2. S_div (Eq. 2, 3) of the CTA's candidates, read in coalesced order
+    //    and staged where the raw votes were, and its extrema over the
+    //    cluster
     float mnD = INFINITY, mxD = -INFINITY;
-  #pragma unroll
-    for (int j = 0; j < kJ; ++j) {
-      const int i = span0 + 32 * j + lane;
-      if (i < Tv) {
-        const float sd = sdiv_rcp(e_[j], c_[j], mnE, invE, f.alpha, mix);
-        mnD = fminf(mnD, sd);
-        mxD = fmaxf(mxD, sd);
+    {
+      const float* dEu = f.dE + (size_t)u * Tv;
+      const float* cvu = f.cosv + (size_t)u * Tv;
+  #pragma unroll 8
+      for (int j = 0; j < kJ; ++j) {
+        const int i = lo + kCThreads * j + tid;
+        if (i < Tv) {
+          const float sd = sdiv_rcp(__ldg(dEu + i), __ldg(cvu + i), mnE, invE, f.alpha, mix);
+          sm.raw[pad_idx(i - lo + kHalo)] = sd;
+          mnD = fminf(mnD, sd);
+          mxD = fmaxf(mxD, sd);
+        }
       }
     }
   #pragma unroll
@@ -217,119 +298,109 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       sm.red[warp][7] = mxD;
     }
     __syncthreads();
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
     if (tid == 0) {
       float a0 = sm.red[0][6], a1 = sm.red[0][7];
       for (int w = 1; w < kCWarps; ++w) {
         a0 = fminf(a0, sm.red[w][6]);
         a1 = fmaxf(a1, sm.red[w][7]);
       }
-      sm.ext[0] = a0;
-      sm.ext[1] = a1;
+      push_all<kMaxC>(cl, &sm.ext_all[rank][0], a0, C);
+      push_all<kMaxC>(cl, &sm.ext_all[rank][1], a1, C);
     }
     cl.sync();
     if (tid == 0) {
       float a0 = INFINITY, a1 = -INFINITY;
       for (int r = 0; r < C; ++r) {
-        const float* pe = cl.map_shared_rank(sm.ext, r);
-        a0 = fminf(a0, pe[0]);
-        a1 = fmaxf(a1, pe[1]);
+        a0 = fminf(a0, sm.ext_all[r][0]);
+        a1 = fmaxf(a1, sm.ext_all[r][1]);
       }
       const float denD = __fadd_rn(__fsub_rn(a1, a0), f.eps);
-      // means: sum_i S_imp(i) = (1/kp) sum_j raw(j) cnt(j), where cnt(j) = kp
-      // except within kp/2 of either end; mean(Sbar) is affine in the means of
-      // d_E and of the cosine (as finalize_unit)
-      const int h = hpool;
-      double edge = 0.0;
-      if (pool_smem) {
-        // sm.edge[l] = raw[l] for l < h, raw[Tv - 2h + l] for h <= l < 2h
-        for (int j = 0; j < Tv && j < h; ++j) edge += (double)sm.edge[j] * (double)(h - j);
-        for (int j = (Tv - h > 0 ? Tv - h : 0); j < Tv; ++j)
-          edge += (double)sm.edge[j - Tv + 2 * h] * (double)(h - (Tv - 1 - j));
-      } else {
-        for (int j = 0; j < Tv && j < h; ++j) edge += (double)__ldg(raw + j) * (double)(h - j);
-        for (int j = (Tv - h > 0 ? Tv - h : 0); j < Tv; ++j) edge += (double)__ldg(raw + j) * (double)(h - (Tv - 1 - j));
-      }
-      const double sum_imp = ((double)f.pool * (double)sm.sc[5] - edge) / (double)f.pool;
-      const double mean_imp = Tv > 0 ? sum_imp / Tv : 0.0;
-      const double mean_sE = Tv > 0 ? ((double)sm.sc[3] / Tv - (double)mnE) / (double)denE : 0.0;
-      const double mean_cs = Tv > 0 ? (double)sm.sc[4] / Tv : 0.0;
-      const double mean_sC = mix ? -mean_cs : (1.0 - mean_cs) * 0.5;
-      const double mean_div = (double)f.alpha * mean_sE + (1.0 - (double)f.alpha) * mean_sC;
-      const double mean_sbar = (mean_div - (double)a0) / (double)denD;
+      // mean(S_imp) / mean(Sbar) with Sbar = (S_div - a0) / denD
+      const double num = sm.dsc[1] - (double)a0 * (double)Tv;  // Tv * denD * mean(Sbar)
       sm.sc[6] = a0;
       sm.sc[7] = denD;
-      sm.sc[5] = mean_sbar > 0.0 ? (float)(mean_imp / mean_sbar) : 0.f;
+      sm.sc[5] = (Tv > 0 && num > 0.0) ? (float)(sm.dsc[0] * (double)denD / ((double)f.pool * num)) : 0.f;
     }
     __syncthreads();
-    const float mnD2 = sm.sc[6], denD = sm.sc[7], scale = sm.sc[5];
+    const float lamf = sm.sc[0], mnD2 = sm.sc[6], denD = sm.sc[7], scale = sm.sc[5];
     const float invD = __frcp_rn(denD);
     const float one_m_lam = __fsub_rn(1.f, lamf);
 
-    // 3. final scores (Eq. 7); the order-preserving keys replace the pooled
-    //    importance in buf
-    float* Sg = f.S ? f.S + (size_t)u * Tv : nullptr;
+    // 3. final scores (Eq. 7); the keys replace the pooled importance, and
+    //    the scores go out through the staging buffer in coalesced order
     float* dbg = f.dbg ? f.dbg + (size_t)u * 5 * Tv : nullptr;
   #pragma unroll
-    for (int j = 0; j < kJ; ++j) {
-      const int i = span0 + 32 * j + lane;
-      if (i < Tv) {
-        const float e = e_[j], c = c_[j];
-        const float sd = sdiv_rcp(e, c, mnE, invE, f.alpha, mix);
-        const float sbar = __fmul_rn(__fsub_rn(sd, mnD2), invD);
-        const float sp = __uint_as_float(sm.buf[i - lo]);
-        const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
-        sm.buf[i - lo] = ordered_key(S);
-        if (Sg) Sg[i] = S;
-        if (dbg) {
-          dbg[i] = __ldg(raw + i);
-          dbg[Tv + i] = sp;
-          dbg[2 * Tv + i] = e;
-          dbg[3 * Tv + i] = c;
-          dbg[4 * Tv + i] = sd;
-        }
+    for (int c = 0; c < kJ; ++c) {
+      const float sd = sm.raw[pad_idx(q0 + c)];
+      const float sbar = __fmul_rn(__fsub_rn(sd, mnD2), invD);
+      const float sp = __uint_as_float(key[c]);
+      const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
+      key[c] = ordered_key(S);
+      sm.raw[pad_idx(q0 + c)] = S;
+      if (dbg && c < nv) {
+        const int i = c0 + c;
+        dbg[i] = __ldg(raw + i);
+        dbg[Tv + i] = sp;
+        dbg[2 * Tv + i] = __ldg(f.dE + (size_t)u * Tv + i);
+        dbg[3 * Tv + i] = __ldg(f.cosv + (size_t)u * Tv + i);
+        dbg[4 * Tv + i] = sd;
+      }
+    }
+    if (f.S != nullptr) {
+      __syncthreads();
+      float* Sg = f.S + (size_t)u * Tv;
+  #pragma unroll 8
+      for (int j = 0; j < kJ; ++j) {
+        const int i = lo + kCThreads * j + tid;
+        if (i < Tv) Sg[i] = sm.raw[pad_idx(i - lo + kHalo)];
       }
     }
   }
 
   if (kSelect) {
-    // 4. radix select of the k-th largest key over the cluster (each thread
-    //    reads back only the keys it wrote)
+    // 4. radix select of the k-th largest key over the cluster
     unsigned prefix = 0u, mask = 0u;
     int rem = k;
     if (k > 0) {
       int pass = 0;
       for (int shift = 24; shift >= 0; shift -= 8, ++pass) {
-        // each warp counts into its own histogram (no two warps contend for
-        // one address: the keys of a head crowd into few bins), then the
-        // CTA's histogram is their sum
+        // each warp counts into its own histogram, a thread adding runs of
+        // equal bins among its consecutive candidates (neighbouring scores
+        // share their leading bits), then the CTA's histogram is the sum of
+        // its warps'
         unsigned* wh = sm.whist[warp];
 #pragma unroll
         for (int b = lane; b < 256; b += 32) wh[b] = 0u;
         __syncwarp();
-#pragma unroll 4
-        for (int j = 0; j < kJ; ++j) {
-          const int i = span0 + 32 * j + lane;
-          unsigned bin = 0xffffffffu;
-          if (i < Tv) {
-            const unsigned key = sm.buf[i - lo];
-            if ((key & mask) == prefix) bin = (key >> shift) & 255u;
+        unsigned cur = 0u, run = 0u;
+#pragma unroll
+        for (int c = 0; c < kJ; ++c) {
+          if (c < nv && (key[c] & mask) == prefix) {
+            const unsigned bin = (key[c] >> shift) & 255u;
+            if (bin != cur) {
+              if (run) atomicAdd(&wh[cur], run);
+              cur = bin;
+              run = 0u;
+            }
+            ++run;
           }
-          const unsigned peers = __match_any_sync(0xffffffffu, bin);
-          if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(&wh[bin], (unsigned)__popc(peers));
         }
+        if (run) atomicAdd(&wh[cur], run);
         __syncthreads();
-        unsigned* hist = sm.hist[pass & 1];
         {
           unsigned cnt = 0u;  // kCThreads == 256 bins: thread tid sums bin tid
 #pragma unroll
           for (int w = 0; w < kCWarps; ++w) cnt += sm.whist[w][tid];
-          hist[tid] = cnt;
+          push_all<kMaxC>(cl, &sm.hall[pass & 1][rank][tid], cnt, C);
         }
         cl.sync();
         // the cluster's histogram (rank order: deterministic), bin tid; suffix
         // sums from the top bin find the bin holding the rem-th largest key
         unsigned tot = 0u;
-        for (int r = 0; r < C; ++r) tot += cl.map_shared_rank(hist, r)[tid];
+#pragma unroll
+        for (int r = 0; r < kMaxC; ++r)
+          if (r < C) tot += sm.hall[pass & 1][r][tid];
         unsigned suf = tot;  // sum of bins tid .. 32 * warp + 31
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -355,69 +426,71 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
 
     // 5. kept candidates: above the threshold, or equal to it among the first
     //    `rem` equal ones by position, emitted in ascending position
-    const unsigned lt = (1u << lane) - 1u;
     int n_gt = 0, n_eq = 0;
     if (k > 0) {
-#pragma unroll 4
-      for (int j = 0; j < kJ; ++j) {
-        const int i = span0 + 32 * j + lane;
-        const unsigned key = i < Tv ? sm.buf[i - lo] : 0u;
-        n_gt += __popc(__ballot_sync(0xffffffffu, i < Tv && key > thr));
-        n_eq += __popc(__ballot_sync(0xffffffffu, i < Tv && key == thr));
+#pragma unroll
+      for (int c = 0; c < kJ; ++c)
+        if (c < nv) {
+          n_gt += key[c] > thr;
+          n_eq += key[c] == thr;
+        }
+    }
+    // exclusive prefix over the threads of the CTA (position order)
+    int gi = n_gt, ei = n_eq;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int yg = __shfl_up_sync(0xffffffffu, gi, o), ye = __shfl_up_sync(0xffffffffu, ei, o);
+      if (lane >= o) {
+        gi += yg;
+        ei += ye;
       }
     }
-    if (lane == 0) {
-      sm.shi[8 + warp] = n_gt;
-      sm.shi[16 + warp] = n_eq;
+    if (lane == 31) {
+      sm.wscan[warp][0] = gi;
+      sm.wscan[warp][1] = ei;
     }
     __syncthreads();
+    int gt_excl = gi - n_gt, eq_excl = ei - n_eq;
+    for (int w = 0; w < warp; ++w) {
+      gt_excl += sm.wscan[w][0];
+      eq_excl += sm.wscan[w][1];
+    }
     if (tid == 0) {
       int g = 0, q = 0;
       for (int w = 0; w < kCWarps; ++w) {
-        g += sm.shi[8 + w];
-        q += sm.shi[16 + w];
+        g += sm.wscan[w][0];
+        q += sm.wscan[w][1];
       }
-      sm.cnt[0] = g;
-      sm.cnt[1] = q;
+      push_all<kMaxC>(cl, &sm.cnt_all[rank][0], g, C);
+      push_all<kMaxC>(cl, &sm.cnt_all[rank][1], q, C);
     }
     cl.sync();
     // candidates kept by lower ranks, and the ties they took
     int pos = 0, eq_before = 0;
     for (int r = 0; r < rank; ++r) {
-      const int* pc = cl.map_shared_rank(sm.cnt, r);
-      const int g = pc[0], q = pc[1];
-      const int tq = max(0, min(q, rem - eq_before));
-      pos += g + tq;
+      const int g = sm.cnt_all[r][0], q = sm.cnt_all[r][1];
+      pos += g + max(0, min(q, rem - eq_before));
       eq_before += q;
     }
-    // within the CTA: warps in order
-    int w_eq_before = eq_before, w_pos = pos;
-    for (int w = 0; w < warp; ++w) {
-      const int q = sm.shi[16 + w];
-      const int tq = max(0, min(q, rem - w_eq_before));
-      w_pos += sm.shi[8 + w] + tq;
-      w_eq_before += q;
-    }
-    const int take_eq = max(0, min(n_eq, rem - w_eq_before));
+    // ties still to take from this CTA on, in position order
+    const int ties = max(0, rem - eq_before);
+    int p = pos + gt_excl + min(ties, eq_excl);
+    int take_eq = max(0, min(n_eq, ties - eq_excl));
     int32_t* out = f.idx + (size_t)u * f.n_keep;
-    int eq_seen = 0;
     if (k > 0) {
-#pragma unroll 4
-      for (int j = 0; j < kJ; ++j) {
-        const int i = span0 + 32 * j + lane;
-        const unsigned key = i < Tv ? sm.buf[i - lo] : 0u;
-        const bool gt = i < Tv && key > thr;
-        const bool eq = i < Tv && key == thr;
-        const unsigned eqm = __ballot_sync(0xffffffffu, eq);
-        const bool take = gt || (eq && eq_seen + __popc(eqm & lt) < take_eq);
-        const unsigned sel = __ballot_sync(0xffffffffu, take);
-        if (take) {
-          const int p = w_pos + __popc(sel & lt);
-          if (p < k) out[p] = i;
+#pragma unroll
+      for (int c = 0; c < kJ; ++c)
+        if (c < nv) {
+          bool take = key[c] > thr;
+          if (!take && key[c] == thr && take_eq > 0) {
+            take = true;
+            --take_eq;
+          }
+          if (take) {
+            if (p < k) out[p] = c0 + c;
+            ++p;
+          }
         }
-        w_pos += __popc(sel);
-        eq_seen += __popc(eqm);
-      }
     }
     if (keep_all) {
       // B >= N: every row in order; rank r writes its candidates, the last rank the window
@@ -429,37 +502,30 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       for (int j = tid; j < f.W; j += kCThreads) out[k + j] = Tv + j;
     }
   }
-  cl.sync();  // no CTA leaves while a peer may still read its shared memory
+  // No CTA touches a peer's shared memory after the last cluster barrier it
+  // passed (every exchange is a store made before that barrier), so the
+  // CTAs may leave independently.
 }
 
-}  // namespace
+template <int kJ>
+cudaError_t set_smem_attrs() {
+  const int bytes = (int)sizeof(ClusterSmem<kJ>);
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                bytes)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                bytes)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(finalize_cluster_kernel<2, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
 
-// Scores (and with f.idx the top-k) of every unit, or with select_only the
-// top-k of the scores in f.S; one cluster per unit; cudaErrorNotSupported
-// when Tv exceeds what eight CTAs hold.
-cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only, cudaStream_t s) {
-  const int C = f.Tv <= 0 ? 1 : (f.Tv + kCap - 1) / kCap;
-  if (C > kMaxCluster) return cudaErrorNotSupported;
-  static bool attr_set[64] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!attr_set[dev]) {
-    const int bytes = (int)sizeof(ClusterSmem);
-    if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  bytes)) != cudaSuccess ||
-        (e = cudaFuncSetAttribute(finalize_cluster_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  bytes)) != cudaSuccess ||
-        (e = cudaFuncSetAttribute(finalize_cluster_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  bytes)) != cudaSuccess)
-      return e;
-    attr_set[dev] = true;
-  }
+template <int kJ>
+cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cudaStream_t s) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)(U * C), 1, 1);
   cfg.blockDim = dim3(kCThreads, 1, 1);
-  cfg.dynamicSmemBytes = sizeof(ClusterSmem);
+  cfg.dynamicSmemBytes = sizeof(ClusterSmem<kJ>);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -468,9 +534,32 @@ cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only,
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2>, f);
-  if (f.idx == nullptr) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0>, f);
-  return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1>, f);
+  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ>, f);
+  if (f.idx == nullptr) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ>, f);
+  return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ>, f);
+}
+
+}  // namespace
+
+// Scores (and with f.idx the top-k) of every unit, or with select_only the
+// top-k of the scores in f.S; one cluster per unit; cudaErrorNotSupported
+// when Tv exceeds what eight CTAs of 4096 (or four of 8192) candidates hold.
+cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only, cudaStream_t s) {
+  const int Tv = f.Tv > 0 ? f.Tv : 1;
+  const int C16 = (Tv + Shape<16>::kCap - 1) / Shape<16>::kCap;
+  const int C32 = (Tv + Shape<32>::kCap - 1) / Shape<32>::kCap;
+  const bool wide = C16 > 4;
+  if (wide ? C32 > Shape<32>::kMaxCluster : C16 > Shape<16>::kMaxCluster) return cudaErrorNotSupported;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!attr_set[dev]) {
+    if ((e = set_smem_attrs<16>()) != cudaSuccess || (e = set_smem_attrs<32>()) != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  return wide ? launch_shape<32>(f, U, C32, select_only, s) : launch_shape<16>(f, U, C16, select_only, s);
 }
 
 }  // namespace ecokv

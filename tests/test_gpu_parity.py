@@ -116,9 +116,19 @@ def test_config_c2_two_layers():
     run_and_compare(CONFIGS["c2"], layers=range(5, 7))
 
 
+@pytest.mark.parametrize("pool_kernel", [5, 7, 41])
+def test_wide_cluster_ragged(pool_kernel):
+    # 20000 candidates: three CTAs of 8192 in a cluster, the last one ragged;
+    # kernel 41 pools from global memory instead of the shared halo
+    w = small_workload(n=20000, h_kv=2, group=4, window=8, budget=2000, pool_kernel=pool_kernel, dtype="bf16",
+                       clustered=True, seed=pool_kernel)
+    run_and_compare(w)
+
+
+# (32768, 8): the finalize takes clusters of four CTAs of 8192 candidates;
 # (65536, 4): more candidates than one thread-block cluster holds, so the
 # finalize runs one CTA per head
-@pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4), (65536, 4)])
+@pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4), (32768, 8), (65536, 4)])
 def test_sweep_points(n, window):
     run_and_compare(sweep_workload(n, window))
 
@@ -153,7 +163,8 @@ def test_identical_keys_all_ties():
         check_rows(Kd[0, 0], idx[0, 0], Ko[0, 0])
 
 
-@pytest.mark.parametrize("n,window,budget", [(5000, 4, 300), (300, 1, 299), (70000, 8, 7000)])
+@pytest.mark.parametrize("n,window,budget", [(5000, 4, 300), (300, 1, 299), (20000, 8, 2000), (32768, 4, 30000),
+                                             (70000, 8, 7000)])
 def test_select_exact_on_crafted_scores(n, window, budget):
     # ties, negatives, +-0: radix select must equal (S desc, position asc)
     g = torch.Generator().manual_seed(n)
