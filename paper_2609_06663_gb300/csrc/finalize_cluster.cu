@@ -105,6 +105,11 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   // The peers must have started before the first store into their shared
   // memory: this arrival is waited for just before it.
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+  // Launched as a programmatic dependent of the streaming pass: let the gather
+  // be scheduled behind this grid, and wait for the previous grid's results
+  // (a no-op when launched plainly).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int C = (int)cl.num_blocks();
   const int rank = (int)cl.block_rank();
   const int u = blockIdx.x / C;
@@ -527,13 +532,15 @@ cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cud
   cfg.blockDim = dim3(kCThreads, 1, 1);
   cfg.dynamicSmemBytes = sizeof(ClusterSmem<kJ>);
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ>, f);
   if (f.idx == nullptr) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ>, f);
   return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ>, f);

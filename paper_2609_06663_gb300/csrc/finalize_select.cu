@@ -31,6 +31,9 @@ __global__ void __launch_bounds__(kFinThreads) select_kernel(FinalArgs f) {
 
 template <typename T>
 __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a) {
+  // launched as a programmatic dependent: the indices come from the previous
+  // grid (a no-op when launched plainly)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   constexpr int rows = 32;
   const int r0 = blockIdx.x * rows;
   gather_rows<T>(a, blockIdx.y, r0, r0 + rows, threadIdx.x, blockDim.x);
@@ -63,12 +66,17 @@ cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s) {
 
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s) {
   if (a.n_keep == 0 || U == 0) return cudaSuccess;
-  const dim3 grid((a.n_keep + 31) / 32, U);
-  if (dt == ECOKV_F32)
-    compact_kernel<float><<<grid, 256, 0, s>>>(a);
-  else
-    compact_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((a.n_keep + 31) / 32, U);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (dt == ECOKV_F32) return cudaLaunchKernelEx(&cfg, compact_kernel<float>, a);
+  return cudaLaunchKernelEx(&cfg, compact_kernel<__nv_bfloat16>, a);
 }
 
 }  // namespace ecokv

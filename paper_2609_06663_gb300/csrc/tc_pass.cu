@@ -725,7 +725,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.item_full[slot]);
       ++seq;
-      if (it.type == kExit) break;
+      if (it.type == kExit) {
+        // no work left for this CTA: the next launch (finalisation) may be
+        // scheduled on SMs as they drain; it waits for this grid's completion
+        // before reading anything
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        break;
+      }
       for (int t = 0; t < ntiles && ok; ++t) {
         if (lane == 0) {
           ok = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
