@@ -20,7 +20,7 @@ namespace ecokv {
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-Layout make_layout(const ecokv_params& p, int chunk) {
+Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
   Layout L{};
   L.U = p.n_layers * p.h_kv;
   L.R = (p.h_q / p.h_kv) * p.window;
@@ -29,6 +29,7 @@ Layout make_layout(const ecokv_params& p, int chunk) {
   L.Tv = p.n - p.window;
   L.chunk = chunk;
   L.nchunks = (p.n + chunk - 1) / chunk;
+  L.p2slots = p2slots;
   L.p1_stride = 2 * ((L.R + 3) & ~3) + 2 * kD;
   L.ustat_stride = (ustat_lse() + L.R + 3) & ~3;
   const size_t U = (size_t)L.U;
@@ -37,7 +38,7 @@ Layout make_layout(const ecokv_params& p, int chunk) {
   L.sync = off;    L.sync_bytes = (4 + 4 * U) * 4;  off += align256(L.sync_bytes);
   L.p1part = off;  off += align256(U * L.nchunks * L.p1_stride * 4);
   L.ustat = off;   off += align256(U * L.ustat_stride * 4);
-  L.p2part = off;  off += align256(U * L.nchunks * kP2Stride * 4);
+  L.p2part = off;  off += align256(U * L.nchunks * L.p2slots * kP2Stride * 4);
   L.simp = off;    off += align256(U * L.Tv * 4);
   L.dE = off;      off += align256(U * L.Tv * 4);
   L.cosv = off;    off += align256(U * L.Tv * 4);
@@ -50,7 +51,7 @@ Layout make_layout(const ecokv_params& p, int chunk) {
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 static size_t workspace_bytes(const ecokv_params& p) {
-  const size_t a = make_layout(p, kChunk).total, b = make_layout(p, kTcChunk).total;
+  const size_t a = make_layout(p, kChunk).total, b = make_layout(p, kTcChunk, kTcP2Parts).total;
   return a > b ? a : b;
 }
 
@@ -90,6 +91,19 @@ static int tc_tiles(const ecokv_params& p) {
 }
 static int tc_chunk_keys(const ecokv_params& p) { return 128 * tc_tiles(p); }
 
+// SMs of the current device (cached per device).
+static int num_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
 static int env_int(const char* name, int dflt, int lo, int hi) {
   const char* v = getenv(name);
   if (v == nullptr || *v == 0) return dflt;
@@ -127,7 +141,7 @@ static FinalArgs final_args(const ecokv_params& p, const Layout& L, char* ws) {
   f.N = p.n;
   f.W = p.window;
   f.Tv = L.Tv;
-  f.nchunks = L.nchunks;
+  f.nchunks = L.nchunks * L.p2slots;
   f.budget = p.budget;
   f.pool = p.pool_kernel;
   f.ustat_stride = L.ustat_stride;
@@ -166,7 +180,7 @@ static CompactArgs compact_args(const ecokv_params& p, const void* K, const void
 // the per-call counters).
 static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
   const int tiles = tc_tiles(p);
-  const Layout L = make_layout(p, 128 * tiles);
+  const Layout L = make_layout(p, 128 * tiles, kTcP2Parts);
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   TcArgs a{};
   a.U = L.U;
@@ -188,7 +202,17 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   // than the items in flight, so nothing is lost (ECOKV_LAG_P2 for tuning)
   a.lag_p2 = env_int("ECOKV_LAG_P2", 1 << 20, 1, 1 << 20);
   if (a.lag_p2 > L.U) a.lag_p2 = L.U;
-  a.total_tickets = 2 * L.U * a.nchunks;
+  // the pass-2 items of the last schedule steps are split in parts, so that
+  // the persistent CTAs run out of work at nearly the same time (the work
+  // after the last ticket is a part, not a whole item); only the steps that
+  // hold pass-2 items alone (the last lag_p2) are eligible
+  const int tail_items = a.lag_p2 * a.nchunks;
+  int nsplit = env_int("ECOKV_TAIL_SPLIT", num_sms(), 0, 1 << 30);
+  if (nsplit > tail_items) nsplit = tail_items;
+  a.nparts = env_int("ECOKV_TAIL_PARTS", kTcP2Parts, 1, kTcP2Parts);
+  if (tiles < a.nparts) a.nparts = tiles;
+  a.split_from = 2 * L.U * a.nchunks - nsplit;
+  a.total_tickets = a.split_from + a.nparts * nsplit;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
@@ -218,8 +242,6 @@ static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const
   return ECOKV_OK;
 }
 
-// Scores (and the top-k) of every unit: one cluster per unit when the unit
-// fits eight CTAs, one CTA per unit otherwise.  Both give the same bits.
 // Scores (and the top-k) of every unit: one cluster per unit when the unit
 // fits eight CTAs, one CTA per unit otherwise.
 static ecokv_status run_finalize(FinalArgs f, int U, bool do_select, cudaStream_t s) {
@@ -285,7 +307,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.lambda = lambda;
@@ -350,7 +372,7 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);

@@ -45,13 +45,14 @@ struct Layout {
   int N, W, Tv;      // tokens, window, candidates
   int chunk;         // keys per streaming chunk
   int nchunks;       // ceil(N / chunk)
+  int p2slots;       // pass-2 partial slots per chunk (a chunk's pass-2 item may be split in parts)
   int p1_stride;     // floats per (unit, chunk) pass-1 partial: 2R + 2D
   int ustat_stride;  // floats per unit statistics record
   size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2, total;
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
 
-Layout make_layout(const ecokv_params& p, int chunk);
+Layout make_layout(const ecokv_params& p, int chunk, int p2slots = 1);
 
 // unit statistics record (floats):  [0,D) kbar | [D,2D) mu | [2D] ||kbar||^2 |
 //                                    [2D+1] ||mu||^2 | [2D+2, 2D+2+R) log2-LSE of the window rows
@@ -80,7 +81,7 @@ struct FinalArgs {
   float alpha, beta, tau, eps, lambda_override;
   unsigned flags;
   int n_keep;
-  const float* p2part;  // [U][nchunks][kP2Stride]
+  const float* p2part;  // [U][nchunks][kP2Stride]: nchunks counts every pass-2 partial slot
   const float* ustat;
   const float* simp;
   const float* dE;

@@ -143,6 +143,22 @@ __device__ bool wait_bar(uint64_t* bar, uint32_t parity, const TcArgs& a, unsign
   }
 }
 
+// Tiles of a chunk, and of part p (1..nparts) of it (its first tile in *t0);
+// part 0 is the whole chunk.
+__device__ __forceinline__ int chunk_tiles(const TcArgs& a, int chunk) {
+  return min(a.tiles_per_chunk, (a.N - chunk * a.tiles_per_chunk * kTile + kTile - 1) / kTile);
+}
+__device__ __forceinline__ int part_tiles(const TcArgs& a, int chunk, int part, int* t0) {
+  const int nt = chunk_tiles(a, chunk);
+  if (part == 0) {
+    if (t0) *t0 = 0;
+    return nt;
+  }
+  const int per = (nt + a.nparts - 1) / a.nparts, first = (part - 1) * per;
+  if (t0) *t0 = first;
+  return min(per, nt - first);
+}
+
 struct Item {
   int type, u, chunk, part;
   bool valid;
@@ -156,6 +172,14 @@ struct Item {
 __device__ Item decode(int ticket, const TcArgs& a) {
   Item it{kExit, 0, 0, 0, true};
   if (ticket >= a.total_tickets) return it;
+  int part = 0;
+  if (ticket >= a.split_from) {
+    // the last pass-2 items, each split in nparts consecutive parts
+    const int rel = ticket - a.split_from;
+    part = 1 + rel % a.nparts;
+    ticket = a.split_from + rel / a.nparts;
+  }
+  it.part = part;
   const int nc = a.nchunks, L = a.lag_p2;
   const int head = L * nc, body = (a.U - L) * 2 * nc;
   if (ticket < head) {
@@ -180,6 +204,7 @@ __device__ Item decode(int ticket, const TcArgs& a) {
     it.chunk = rel - v * nc;
   }
   it.valid = it.u >= 0 && it.u < a.U;
+  if (part > 0 && part_tiles(a, it.chunk, part, nullptr) <= 0) it.valid = false;  // a part past the chunk's end
   return it;
 }
 
@@ -661,8 +686,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float x = s.red6[w4][tid];
             acc = tid == 1 ? fminf(acc, x) : tid == 2 ? fmaxf(acc, x) : acc + x;
           }
-          float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kP2Stride;
-          p[tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
+          // the chunk's slot of this part; the first part also fills every
+          // slot no part writes with the identity of its reduction
+          float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kTcP2Parts * kP2Stride;
+          const int part = d.part;
+          p[(part > 0 ? part - 1 : 0) * kP2Stride + tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
+          if (part <= 1) {
+            const float idn = tid == P2_MIN_DE ? INFINITY : tid == P2_MAX_DE ? -INFINITY : 0.f;
+            for (int q = 1; q < kTcP2Parts; ++q)
+              if (part == 0 || q >= a.nparts || part_tiles(a, chunk, q + 1, nullptr) <= 0) p[q * kP2Stride + tid] = idn;
+          }
         }
       }
       __syncwarp();
@@ -694,8 +727,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
       if (!ok) break;
       ItemDesc& d = s.desc[slot];
-      const int i0 = it.chunk * a.tiles_per_chunk * kTile;
-      const int ntiles = it.type == kExit ? 0 : min(a.tiles_per_chunk, (a.N - i0 + kTile - 1) / kTile);
+      int t0 = 0;
+      const int ntiles = it.type == kExit ? 0 : part_tiles(a, it.chunk, it.part, &t0);
+      const int i0 = (it.chunk * a.tiles_per_chunk + t0) * kTile;
       if (lane == 0) {
         d.type = it.type;
         d.u = it.u;

@@ -8,13 +8,16 @@ namespace ecokv {
 constexpr int kTcMaxTiles = 64;                // largest item: 64 tiles of 128 keys
 constexpr int kTcMinTiles = 2;                 // smallest item the workspace is sized for
 constexpr int kTcChunk = 128 * kTcMinTiles;
+constexpr int kTcP2Parts = 4;                  // parts a tail pass-2 item is split into (its partial slots)
 
 struct TcArgs {
   int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
   int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
   int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1 (<= U)
-  int total_tickets;                // 2 * U * nchunks
+  int split_from;                   // tickets from here on: pass-2 items split in nparts parts
+  int nparts;                       // 1 .. kTcP2Parts
+  int total_tickets;                // split_from + nparts * (2 * U * nchunks - split_from)
   int p1_stride, ustat_stride;
   float scale_log2;
   long long timeout_cycles;
@@ -23,7 +26,7 @@ struct TcArgs {
   float* norm2;                     // [U][N] squared key norms written by pass 1
   float* p1part;
   float* ustat;
-  float* p2part;
+  float* p2part;                    // [U][nchunks][kTcP2Parts][kP2Stride]
   float* simp;
   float* dE;
   float* cosv;
