@@ -126,6 +126,9 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   const bool pool_smem = hpool <= kHalo;
   const float* us = f.ustat + (size_t)u * f.ustat_stride;
   const float* raw = f.simp + (size_t)u * Tv;
+  // the per-candidate arrays of this unit start 16-byte aligned: sweeps in
+  // groups of four
+  const bool vec4 = ((u * Tv) & 3) == 0;
 
   // pooled importance (as float bits), then the order-preserving keys of S
   unsigned key[kJ];
@@ -159,11 +162,33 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       v6[4] += __ldg(p + P2_SUM_COS);
       v6[5] += __ldg(p + P2_SUM_RAW);
     }
-    if (pool_smem)
-      for (int q = kHalo - hpool + tid; q < kHalo + kCap + hpool; q += kCThreads) {
-        const int j = lo - kHalo + q;
-        sm.raw[pad_idx(q)] = (j >= 0 && j < Tv) ? __ldg(raw + j) : 0.f;
+    if (pool_smem) {
+      if (vec4) {
+        // the whole halo of kHalo each side in 16-byte loads (kHalo and lo are
+        // multiples of four, so each group of four lies inside [0, Tv) or
+        // outside it entirely except at the ragged end)
+        for (int q = 4 * tid; q < kCap + 2 * kHalo; q += 4 * kCThreads) {
+          const int j = lo - kHalo + q;
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (j >= 0 && j + 3 < Tv) {
+            v = __ldg(reinterpret_cast<const float4*>(raw + j));
+          } else if (j >= 0 && j < Tv) {
+            v.x = __ldg(raw + j);
+            if (j + 1 < Tv) v.y = __ldg(raw + j + 1);
+            if (j + 2 < Tv) v.z = __ldg(raw + j + 2);
+          }
+          sm.raw[pad_idx(q)] = v.x;
+          sm.raw[pad_idx(q + 1)] = v.y;
+          sm.raw[pad_idx(q + 2)] = v.z;
+          sm.raw[pad_idx(q + 3)] = v.w;
+        }
+      } else {
+        for (int q = kHalo - hpool + tid; q < kHalo + kCap + hpool; q += kCThreads) {
+          const int j = lo - kHalo + q;
+          sm.raw[pad_idx(q)] = (j >= 0 && j < Tv) ? __ldg(raw + j) : 0.f;
+        }
       }
+    }
     if (warp == 1 && lane < 2 * hpool && pool_smem) {
       const int j = lane < hpool ? lane : Tv - 2 * hpool + lane;
       sm.edge[lane] = (j >= 0 && j < Tv) ? __ldg(raw + j) : 0.f;
@@ -282,14 +307,43 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     {
       const float* dEu = f.dE + (size_t)u * Tv;
       const float* cvu = f.cosv + (size_t)u * Tv;
+      if (vec4) {
+  #pragma unroll 4
+        for (int j = 0; j < kJ / 4; ++j) {
+          const int i = lo + 4 * (kCThreads * j + tid);
+          if (i < Tv) {
+            float e[4] = {0.f, 0.f, 0.f, 0.f}, cs[4] = {0.f, 0.f, 0.f, 0.f};
+            if (i + 3 < Tv) {
+              const float4 a4 = __ldg(reinterpret_cast<const float4*>(dEu + i));
+              const float4 b4 = __ldg(reinterpret_cast<const float4*>(cvu + i));
+              e[0] = a4.x; e[1] = a4.y; e[2] = a4.z; e[3] = a4.w;
+              cs[0] = b4.x; cs[1] = b4.y; cs[2] = b4.z; cs[3] = b4.w;
+            } else {
+              for (int r = 0; r < 4 && i + r < Tv; ++r) {
+                e[r] = __ldg(dEu + i + r);
+                cs[r] = __ldg(cvu + i + r);
+              }
+            }
+  #pragma unroll
+            for (int r = 0; r < 4; ++r)
+              if (i + r < Tv) {
+                const float sd = sdiv_rcp(e[r], cs[r], mnE, invE, f.alpha, mix);
+                sm.raw[pad_idx(i + r - lo + kHalo)] = sd;
+                mnD = fminf(mnD, sd);
+                mxD = fmaxf(mxD, sd);
+              }
+          }
+        }
+      } else {
   #pragma unroll 8
-      for (int j = 0; j < kJ; ++j) {
-        const int i = lo + kCThreads * j + tid;
-        if (i < Tv) {
-          const float sd = sdiv_rcp(__ldg(dEu + i), __ldg(cvu + i), mnE, invE, f.alpha, mix);
-          sm.raw[pad_idx(i - lo + kHalo)] = sd;
-          mnD = fminf(mnD, sd);
-          mxD = fmaxf(mxD, sd);
+        for (int j = 0; j < kJ; ++j) {
+          const int i = lo + kCThreads * j + tid;
+          if (i < Tv) {
+            const float sd = sdiv_rcp(__ldg(dEu + i), __ldg(cvu + i), mnE, invE, f.alpha, mix);
+            sm.raw[pad_idx(i - lo + kHalo)] = sd;
+            mnD = fminf(mnD, sd);
+            mxD = fmaxf(mxD, sd);
+          }
         }
       }
     }
@@ -355,10 +409,24 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     if (f.S != nullptr) {
       __syncthreads();
       float* Sg = f.S + (size_t)u * Tv;
+      if (vec4) {
+  #pragma unroll 4
+        for (int j = 0; j < kJ / 4; ++j) {
+          const int i = lo + 4 * (kCThreads * j + tid);
+          const int q = i - lo + kHalo;
+          if (i + 3 < Tv) {
+            *reinterpret_cast<float4*>(Sg + i) =
+                make_float4(sm.raw[pad_idx(q)], sm.raw[pad_idx(q + 1)], sm.raw[pad_idx(q + 2)], sm.raw[pad_idx(q + 3)]);
+          } else {
+            for (int r = 0; r < 4 && i + r < Tv; ++r) Sg[i + r] = sm.raw[pad_idx(q + r)];
+          }
+        }
+      } else {
   #pragma unroll 8
-      for (int j = 0; j < kJ; ++j) {
-        const int i = lo + kCThreads * j + tid;
-        if (i < Tv) Sg[i] = sm.raw[pad_idx(i - lo + kHalo)];
+        for (int j = 0; j < kJ; ++j) {
+          const int i = lo + kCThreads * j + tid;
+          if (i < Tv) Sg[i] = sm.raw[pad_idx(i - lo + kHalo)];
+        }
       }
     }
   }
@@ -424,7 +492,8 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         prefix |= (unsigned)sm.shi[1] << shift;
         mask |= 255u << shift;
         rem = sm.shi[2];
-        __syncthreads();
+        // (the next write of shi follows the next pass's first barrier, which
+        // every thread reaches only after reading this one)
       }
     }
     const unsigned thr = prefix;
