@@ -388,22 +388,34 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
 
     // 3. final scores (Eq. 7); the keys replace the pooled importance, and
     //    the scores go out through the staging buffer in coalesced order
-    float* dbg = f.dbg ? f.dbg + (size_t)u * 5 * Tv : nullptr;
   #pragma unroll
     for (int c = 0; c < kJ; ++c) {
       const float sd = sm.raw[pad_idx(q0 + c)];
       const float sbar = __fmul_rn(__fsub_rn(sd, mnD2), invD);
-      const float sp = __uint_as_float(key[c]);
-      const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, sp));
+      const float S = __fadd_rn(__fmul_rn(lamf, __fmul_rn(sbar, scale)), __fmul_rn(one_m_lam, __uint_as_float(key[c])));
       key[c] = ordered_key(S);
       sm.raw[pad_idx(q0 + c)] = S;
-      if (dbg && c < nv) {
+    }
+    if (f.dbg != nullptr) {
+      // per-candidate terms for inspection: raw vote, pooled importance, d_E,
+      // cosine, S_div, recomputed by the same operations (kept out of the
+      // loop above, whose code size sets its speed)
+      float* dbg = f.dbg + (size_t)u * 5 * Tv;
+      const float* dEu = f.dE + (size_t)u * Tv;
+      const float* cvu = f.cosv + (size_t)u * Tv;
+      const float inv_pool = __frcp_rn((float)f.pool);
+  #pragma unroll 1
+      for (int c = 0; c < nv; ++c) {
         const int i = c0 + c;
+        float acc = 0.f;
+        for (int o = -hpool; o <= hpool; ++o)
+          if (i + o >= 0 && i + o < Tv) acc = __fadd_rn(acc, __ldg(raw + i + o));
+        const float e = __ldg(dEu + i), cs = __ldg(cvu + i);
         dbg[i] = __ldg(raw + i);
-        dbg[Tv + i] = sp;
-        dbg[2 * Tv + i] = __ldg(f.dE + (size_t)u * Tv + i);
-        dbg[3 * Tv + i] = __ldg(f.cosv + (size_t)u * Tv + i);
-        dbg[4 * Tv + i] = sd;
+        dbg[Tv + i] = __fmul_rn(acc, inv_pool);
+        dbg[2 * Tv + i] = e;
+        dbg[3 * Tv + i] = cs;
+        dbg[4 * Tv + i] = sdiv_rcp(e, cs, mnE, invE, f.alpha, mix);
       }
     }
     if (f.S != nullptr) {
