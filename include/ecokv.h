@@ -159,6 +159,37 @@ ecokv_status ecokv_evict_noalloc(const ecokv_params* p, ecokv_dtype dtype, const
                                  const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
                                  float* lambda, uint32_t* dev_status, void* stream);
 
+/* The whole pass for a KV cache resident in host memory.  The paper has no
+ * counterpart: this is a deployment variant of ecokv_evict for caches kept in
+ * host memory that the GPU can address (e.g. offloaded layers on a
+ * Grace-Blackwell node), where the host link, not the GPU, sets the pace.
+ *
+ * Every host buffer below must be device-accessible at the same address:
+ * pinned with cudaHostAlloc / cudaMallocHost, or registered with
+ * cudaHostRegister(..., cudaHostRegisterMapped), on a system with unified
+ * addressing.  Checked with cudaPointerGetAttributes before anything is
+ * launched (ECOKV_ERR_INVALID_ARG otherwise).
+ *   K, V, Qwin     : host inputs (dtype), layouts as for ecokv_evict.
+ *   idx            : host out, int32 [L][h_kv][min(B, n)].
+ *   K_out, V_out   : host out, [L][h_kv][min(B, n)][d].
+ *   lambda         : host out, float32 [L][h_kv]; may be NULL.
+ *   ws, ws_bytes   : device workspace of at least ecokv_workspace_size_host()
+ *                    bytes, 16-byte aligned; it also holds the device copy of
+ *                    K and Qwin and the indices.
+ * Data movement, in stream order: K and Qwin are copied to the workspace once
+ * (both streaming passes read them there); the gather reads the kept V rows
+ * and writes K_out / V_out directly in host memory, so V crosses the host
+ * link only for the kept rows; idx is copied back at the end.  Per call the
+ * host link carries |K| + |Qwin| + B/n of |V| inbound and |K_out| + |V_out| +
+ * |idx| outbound, against |K| + |V| + |Qwin| inbound for ecokv_evict on
+ * copied inputs.  Returns after enqueueing; the outputs are valid once
+ * `stream` has reached that point.  Scores are not returned (use
+ * ecokv_score on device copies for them). */
+size_t ecokv_workspace_size_host(const ecokv_params* p, ecokv_dtype dtype);
+ecokv_status ecokv_evict_host(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                              const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* lambda,
+                              void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, then read and clear the workspace's device status
  * word.  Returns ECOKV_OK, ECOKV_ERR_DEVICE_INDEX, ECOKV_ERR_TIMEOUT, or
  * ECOKV_ERR_CUDA if the synchronisation itself failed. */

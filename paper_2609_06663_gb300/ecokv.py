@@ -25,7 +25,7 @@ STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED",
 
 EXPORTS = ("ecokv_params_default", "ecokv_check_params", "ecokv_workspace_size", "ecokv_score",
            "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string",
-           "ecokv_evict_noalloc", "ecokv_set_stage_events")
+           "ecokv_evict_noalloc", "ecokv_set_stage_events", "ecokv_workspace_size_host", "ecokv_evict_host")
 
 
 class EcokvError(RuntimeError):
@@ -74,6 +74,10 @@ def lib() -> ctypes.CDLL:
         L.ecokv_evict.restype = ctypes.c_int
         L.ecokv_evict_noalloc.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
         L.ecokv_evict_noalloc.restype = ctypes.c_int
+        L.ecokv_workspace_size_host.argtypes = [_P, ctypes.c_int]
+        L.ecokv_workspace_size_host.restype = _sz
+        L.ecokv_evict_host.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+        L.ecokv_evict_host.restype = ctypes.c_int
         L.ecokv_set_stage_events.argtypes = [ctypes.POINTER(_vp), ctypes.c_int]
         L.ecokv_set_stage_events.restype = ctypes.c_int
         L.ecokv_device_status.argtypes = [_vp, _vp]
@@ -141,6 +145,15 @@ def ecokv_compact(p, dtype, K, V, idx, K_out, V_out, ws=None, ws_bytes=0, stream
 def ecokv_evict(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, ws, ws_bytes, stream=None) -> int:
     return lib().ecokv_evict(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx), _ptr(K_out),
                              _ptr(V_out), _ptr(S), _ptr(lam), _ptr(ws), ws_bytes, _stream(stream))
+
+
+def ecokv_workspace_size_host(p, dtype) -> int:
+    return lib().ecokv_workspace_size_host(ctypes.byref(p), dtype)
+
+
+def ecokv_evict_host(p, dtype, K, V, Qwin, idx, K_out, V_out, lam, ws, ws_bytes, stream=None) -> int:
+    return lib().ecokv_evict_host(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx), _ptr(K_out),
+                                  _ptr(V_out), _ptr(lam), _ptr(ws), ws_bytes, _stream(stream))
 
 
 def ecokv_evict_noalloc(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, dev_status, stream=None) -> int:
@@ -233,6 +246,30 @@ def evict(p, K, V, Qwin, ws=None, want_scores=False, stream=None):
     _check(ecokv_evict(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, ws, ws.numel(), stream),
            "ecokv_evict")
     return idx, Ko, Vo, S, lam
+
+
+def alloc_workspace_host(p, dtype, device="cuda"):
+    """Device workspace for ecokv_evict_host (uint8 tensor)."""
+    import torch
+    n = ecokv_workspace_size_host(p, dtype)
+    if n == 0:
+        raise EcokvError(ECOKV_ERR_INVALID_ARG, "ecokv_workspace_size_host")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def evict_host(p, K, V, Qwin, ws=None, stream=None):
+    """Run ecokv_evict_host on pinned host tensors; returns pinned host
+    (idx, K_out, V_out, lambda), valid once the stream has been synchronised."""
+    import torch
+    dt = dtype_code(K)
+    ws = alloc_workspace_host(p, dt) if ws is None else ws
+    n_keep = min(p.budget, p.n)
+    idx = torch.empty(p.n_layers, p.h_kv, n_keep, dtype=torch.int32).pin_memory()
+    Ko = torch.empty(p.n_layers, p.h_kv, n_keep, p.d, dtype=K.dtype).pin_memory()
+    Vo = torch.empty(p.n_layers, p.h_kv, n_keep, p.d, dtype=K.dtype).pin_memory()
+    lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32).pin_memory()
+    _check(ecokv_evict_host(p, dt, K, V, Qwin, idx, Ko, Vo, lam, ws, ws.numel(), stream), "ecokv_evict_host")
+    return idx, Ko, Vo, lam
 
 
 def evict_noalloc(p, K, V, Qwin, want_scores=False, stream=None):

@@ -85,6 +85,11 @@ def test_entry_points_reject_bad_arguments_before_launch(lib):
     assert E.ecokv_evict(p, 1, fake, fake, fake, fake, fake, fake, None, None, None, 0) == 3
     # bad dtype code
     assert E.ecokv_compact(p, 7, fake, fake, fake, fake, fake) == 1
+    # host entry: pointers the device cannot address (no device here at all)
+    ws_host = E.ecokv_workspace_size_host(p, 1)
+    assert ws_host >= ws_need + 2 * 4 * 4096 * 128 * 2          # holds the device copy of K
+    assert E.ecokv_workspace_size_host(p, 7) == 0
+    assert E.ecokv_evict_host(p, 1, fake, fake, fake, fake, fake, fake, None, fake, ws_host) == 1
     # invalid params win over everything
     p.d = 64
     assert E.ecokv_evict(p, 1, fake, fake, fake, fake, fake, fake, None, None, fake, ws_need) == 2
