@@ -18,7 +18,10 @@ Sec. 5.1-5.2 Eq. 1-7, Appendix A "SnapKV" and "MixKV", Algorithm 1):
   5. S_div = alpha s_E + (1 - alpha) s_C (Eq. 3), lambda = beta r_E +
      (1 - beta) r_C (Eq. 6), diversity rescale (Sec. 5.2), S (Eq. 7);
   6. top-(B - W) of S over the non-window keys plus the whole window
-     (Sec. 3), and the gather of the retained K/V rows.
+     (Sec. 3), and the gather of the retained K/V rows;
+  7. (variant, AdaKV's layer-wide budget, Appendix A) one top-H_kv (B - W)
+     over the concatenated scores of a layer's heads instead of one top-(B - W)
+     per head.
 
 Readings of passages that are silent, ambiguous or garbled (each one is also
 listed with its justification in the design notes):
@@ -51,6 +54,9 @@ listed with its justification in the design notes):
   R13 tau = sqrt(d) unless given; sigma is the logistic function.
   R14 Query head q belongs to KV head q // (h_q / h_kv).
   R15 r_C := 1 when N = 1 (a single key is fully redundant with itself).
+  R16 Layer-wide budget (AdaKV): the layer's candidate budget is H_kv (B - W);
+      ties across heads go to the lower head, then the lower position; every
+      head keeps its whole window.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -232,6 +238,30 @@ def select(S: np.ndarray, p: Params) -> np.ndarray:
     return np.concatenate([chosen, np.arange(t_v, n)]).astype(np.int64)
 
 
+def select_adaptive(S_heads: list, p: Params) -> list:
+    """Layer-wide budget (AdaKV, Appendix A: the heads' scores are concatenated,
+    one top-K is taken over the concatenation, and each head keeps what it got
+    there).  Readings: K = H_kv (B - W), the layer's candidate budget, so the
+    layer keeps H_kv B rows in all; ties go to the lower (head, position); each
+    head's list is its chosen candidates in ascending position, then its window.
+    B >= N keeps every row of every head.  Returns one index array per head."""
+    n, w, t_v = p.n, p.window, p.t_v
+    h_kv = len(S_heads)
+    if p.budget >= n:
+        return [np.arange(n, dtype=np.int64) for _ in range(h_kv)]
+    k_layer = h_kv * (p.budget - w)
+    cat = np.concatenate([np.asarray(s, dtype=np.float64) for s in S_heads])
+    assert cat.shape == (h_kv * t_v,)
+    order = np.lexsort((np.arange(cat.size), -cat))       # primary -S, then (head, position)
+    chosen = np.zeros(cat.size, dtype=bool)
+    chosen[order[:k_layer]] = True
+    out = []
+    for h in range(h_kv):
+        mine = np.nonzero(chosen[h * t_v:(h + 1) * t_v])[0]
+        out.append(np.concatenate([mine, np.arange(t_v, n)]).astype(np.int64))
+    return out
+
+
 def compact(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
     """Gather the retained rows: X_out[r] = X[idx[r]]."""
     return X[idx]
@@ -292,6 +322,24 @@ def to_f64(x) -> np.ndarray:
     if hasattr(x, "detach"):                      # torch tensor, without importing torch
         x = x.detach().cpu().double().numpy()
     return np.asarray(x, dtype=np.float64)
+
+
+def evict_adaptive(K, V, Q, p: Params, layers=None) -> dict:
+    """The pass with the layer-wide budget of select_adaptive.  Returns, per
+    layer l, the per-head score intermediates ('heads'), 'idx' (the heads'
+    lists concatenated in head order), 'head_off' (H_kv + 1 offsets into it)
+    and the gathered 'K_out' / 'V_out' rows in the same order."""
+    K, V, Q = to_f64(K), to_f64(V), to_f64(Q)
+    g = p.group
+    res = {}
+    for l in (layers if layers is not None else range(p.n_layers)):
+        heads = [score_head(K[l, h], Q[l, h * g:(h + 1) * g], p) for h in range(p.h_kv)]
+        lists = select_adaptive([r["S"] for r in heads], p)
+        off = np.concatenate([[0], np.cumsum([len(x) for x in lists])]).astype(np.int64)
+        res[l] = {"heads": heads, "idx": np.concatenate(lists), "head_off": off,
+                  "K_out": np.concatenate([compact(K[l, h], lists[h]) for h in range(p.h_kv)]),
+                  "V_out": np.concatenate([compact(V[l, h], lists[h]) for h in range(p.h_kv)])}
+    return res
 
 
 def evict(K, V, Q, p: Params, heads=None) -> dict:
