@@ -49,6 +49,8 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=0,
                     help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--variant", choices=["per-head", "adaptive"], default="per-head",
+                    help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -308,8 +310,19 @@ def main():
     stream = torch.cuda.current_stream(dev)
     dt = E.dtype_code(K)
 
+    adaptive = args.variant == "adaptive"
+    if adaptive:
+        rows = w.h_kv * n_keep
+        idx_a = torch.empty(w.n_layers, rows, dtype=torch.int32, device=dev)
+        off_a = torch.empty(w.n_layers, w.h_kv + 1, dtype=torch.int32, device=dev)
+        Ko_a = torch.empty(w.n_layers, rows, w.d, dtype=K.dtype, device=dev)
+        Vo_a = torch.empty_like(Ko_a)
+
     def step():
-        code = E.ecokv_evict(p, dt, K, V, Q, idx, Ko, Vo, None, lam, ws, ws.numel(), stream)
+        if adaptive:
+            code = E.ecokv_evict_adaptive(p, dt, K, V, Q, idx_a, off_a, Ko_a, Vo_a, lam, ws, ws.numel(), stream)
+        else:
+            code = E.ecokv_evict(p, dt, K, V, Q, idx, Ko, Vo, None, lam, ws, ws.numel(), stream)
         if code:
             raise E.EcokvError(code, "ecokv_evict")
 
@@ -363,7 +376,7 @@ def main():
     # Consecutive calls alternate between two streams with their own
     # workspaces, so one call's copy-in overlaps the previous call's kernels.
     e2e = None
-    if args.e2e_steps > 0:
+    if args.e2e_steps > 0 and not adaptive:
         hK = K.cpu().pin_memory()
         hV = V.cpu().pin_memory()
         hQ = Q.cpu().pin_memory()
@@ -441,10 +454,12 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
         "data": "synthetic (seeded anisotropic + clustered/temporally correlated keys; no dataset)",
         "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
+                   "variant": "layer-wide budget (ecokv_evict_adaptive)" if adaptive else "per-head budget",
                    "evicted_rows_per_s": round(job_rate(world, w.units * max(0, w.n - w.budget), ms_step), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-        "gpu_launches": launches_per_call(w) * args.steps, "clocks": clocks,
+        # the layer-wide budget adds the layer select (3 digits x 2, count, emit) and the split
+        "gpu_launches": (launches_per_call(w) + (9 if adaptive else 0)) * args.steps, "clocks": clocks,
         "timing": {"headline": f"{args.steps} steps back to back, CUDA events around the region",
                    "stages": f"{args.steps} further steps with per-launch events (launches serialised)",
                    "staged_ms_per_step": round(staged_ms_step, 5)},

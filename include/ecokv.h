@@ -132,6 +132,26 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
                          const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
                          float* lambda, void* ws, size_t ws_bytes, void* stream);
 
+/* The whole pass with a layer-wide budget (AdaKV, Appendix A): instead of
+ * each head keeping its own top-(B - W), the heads of a layer share one
+ * budget of h_kv (B - W) candidates, taken as one top-K over their
+ * concatenated scores (ties to the lower head, then the lower position); each
+ * head keeps its window as well, so every layer keeps h_kv min(B, n) rows in
+ * all, split unevenly between its heads.
+ *   K, V, Qwin : as for ecokv_evict.
+ *   idx        : out, int32 [L][h_kv * min(B, n)]: per layer the heads' lists
+ *                in head order, each its kept candidates in ascending
+ *                position, then its window N - W .. N - 1.
+ *   head_off   : out, int32 [L][h_kv + 1]: head h's list is
+ *                idx[l][head_off[l][h] .. head_off[l][h + 1]).
+ *   K_out, V_out : out, [L][h_kv * min(B, n)][d], the rows idx names, in its order.
+ *   lambda     : out, float32 [L][h_kv]; may be NULL.
+ *   ws         : as for ecokv_evict (the same size).
+ * B >= n keeps every row (head_off[l][h] = h n). */
+ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                                  const void* Qwin, int32_t* idx, int32_t* head_off, void* K_out,
+                                  void* V_out, float* lambda, void* ws, size_t ws_bytes, void* stream);
+
 /* ecokv_evict without a caller workspace and without any allocation.  The
  * paper has no counterpart: this is a deployment variant of the same pass for
  * callers that may not allocate device memory where they evict (a runtime

@@ -44,6 +44,10 @@ Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
   L.cosv = off;    off += align256(U * L.Tv * 4);
   L.sbuf = off;    off += align256(U * L.Tv * 4);
   L.norm2 = off;   off += align256(U * (size_t)L.N * 4);
+  const size_t n_keep = (size_t)(p.budget < p.n ? p.budget : p.n);
+  L.chosen = off;  off += align256(U * n_keep * 4);
+  L.src = off;     off += align256(U * n_keep * 4);
+  L.lsel = off;    off += align256(layer_select_scratch_bytes(p.n_layers, p.h_kv * L.Tv));
   L.total = off;
   return L;
 }
@@ -354,6 +358,64 @@ ecokv_status ecokv_compact(const ecokv_params* p, ecokv_dtype dtype, const void*
   unsigned* status = ws ? reinterpret_cast<unsigned*>(static_cast<char*>(ws) + L.status) : nullptr;
   const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, status);
   if (launch_compact(c, dtype, L.U, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
+  return ECOKV_OK;
+}
+
+ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                                  const void* Qwin, int32_t* idx, int32_t* head_off, void* K_out, void* V_out,
+                                  float* lambda, void* ws, size_t ws_bytes, void* stream) {
+  ecokv_status st = ecokv_check_params(p);
+  if (st != ECOKV_OK) return st;
+  if (dtype != ECOKV_F32 && dtype != ECOKV_BF16) return ECOKV_ERR_INVALID_ARG;
+  if (!K || !V || !Qwin || !idx || !head_off || !K_out || !V_out) return ECOKV_ERR_INVALID_ARG;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(Qwin) || !aligned16(idx) || !aligned16(K_out) ||
+      !aligned16(V_out) || ((uintptr_t)head_off & 3u) || (lambda && ((uintptr_t)lambda & 3u)))
+    return ECOKV_ERR_INVALID_ARG;
+  if ((st = check_ws(p, ws, ws_bytes)) != ECOKV_OK) return st;
+  char* w = static_cast<char*>(ws);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool tc = use_tensor_path(*p, dtype);
+  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
+  const int n_keep = p->budget < p->n ? p->budget : p->n;
+  const bool keep_all = p->budget >= p->n;
+  // 1. every head's scores, into the workspace
+  FinalArgs f = final_args(*p, L, w);
+  f.S = reinterpret_cast<float*>(w + L.sbuf);
+  f.lambda = lambda;
+  stage_event(0, s);
+  st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
+  if (st != ECOKV_OK) return st;
+  stage_event(1, s);
+  if (run_finalize(f, L.U, false, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
+  // 2. one top-h_kv (B - W) per layer over its heads' concatenated scores
+  //    ([h_kv][Tv] per layer is contiguous), ties to the lower (head, position)
+  AdaptArgs a{};
+  a.chosen = reinterpret_cast<const int32_t*>(w + L.chosen);
+  a.idx = idx;
+  a.head_off = head_off;
+  a.src = reinterpret_cast<int32_t*>(w + L.src);
+  a.h_kv = p->h_kv;
+  a.N = p->n;
+  a.W = p->window;
+  a.Tv = L.Tv;
+  a.n_keep = n_keep;
+  a.k_layer = keep_all ? 0 : p->h_kv * (p->budget - p->window);
+  a.keep_all = keep_all ? 1 : 0;
+  if (!keep_all && a.k_layer > 0 &&
+      launch_layer_select(f.S, p->n_layers, p->h_kv * L.Tv, a.k_layer, reinterpret_cast<int32_t*>(w + L.chosen),
+                          w + L.lsel, s) != cudaSuccess)
+    return ECOKV_ERR_CUDA;
+  // 3. per-head lists and offsets, then the gather over each layer's
+  //    [h_kv * N] rows
+  if (launch_adaptive_split(a, p->n_layers, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(2, s);
+  ecokv_params pl = *p;
+  pl.n = p->h_kv * p->n;
+  pl.budget = p->h_kv * n_keep;
+  CompactArgs c = compact_args(pl, K, V, reinterpret_cast<const int32_t*>(w + L.src), K_out, V_out,
+                               reinterpret_cast<unsigned*>(w + L.status));
+  if (launch_compact(c, dtype, p->n_layers, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  stage_event(3, s);
   return ECOKV_OK;
 }
 

@@ -48,7 +48,10 @@ struct Layout {
   int p2slots;       // pass-2 partial slots per chunk (a chunk's pass-2 item may be split in parts)
   int p1_stride;     // floats per (unit, chunk) pass-1 partial: 2R + 2D
   int ustat_stride;  // floats per unit statistics record
-  size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2, total;
+  size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2;
+  size_t chosen, src;  // layer-wide budget: chosen positions, gathered rows (U * min(B, N) int32 each)
+  size_t lsel;         // layer-wide budget: the layer select's histograms, state and block counts
+  size_t total;
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
 
@@ -103,6 +106,18 @@ struct CompactArgs {
   unsigned* status;  // may be null
 };
 
+// Layer-wide budget (AdaKV): the split of each layer's chosen positions into
+// per-head lists (kept candidates ascending, then the window), their offsets,
+// and the rows of the layer's [h_kv * N] block the gather reads.
+struct AdaptArgs {
+  const int32_t* chosen;  // [L][k_layer] ascending positions in the layer's concatenated scores
+  int32_t* idx;           // [L][h_kv * n_keep]
+  int32_t* head_off;      // [L][h_kv + 1]
+  int32_t* src;           // [L][h_kv * n_keep]
+  int h_kv, N, W, Tv, n_keep, k_layer;
+  int keep_all;           // B >= N: every row of every head
+};
+
 // launchers (return cudaGetLastError() after the launch)
 cudaError_t launch_score_simt(const ScoreArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
 // finalize (scores), then optionally select and gather, one CTA per unit
@@ -110,6 +125,11 @@ cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStrea
 // select only, on caller scores f.S
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s);
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
+cudaError_t launch_adaptive_split(const AdaptArgs& a, int n_layers, cudaStream_t s);
+// k largest of each layer's T scores, ascending positions (layer_select.cu)
+size_t layer_select_scratch_bytes(int n_layers, int T);
+cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int32_t* chosen, void* scratch,
+                                cudaStream_t s);
 // One thread-block cluster per unit: scores, and the top-k when f.idx is set
 // (select_only: the top-k of the given scores f.S); cudaErrorNotSupported
 // when the unit is too long for one cluster.

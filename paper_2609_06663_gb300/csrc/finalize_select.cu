@@ -39,7 +39,55 @@ __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a) {
   gather_rows<T>(a, blockIdx.y, r0, r0 + rows, threadIdx.x, blockDim.x);
 }
 
+// One CTA per (head, layer): the head's share of the layer's chosen positions
+// (a contiguous run of the ascending list, found by binary search), written
+// as positions in the head, then its window; the head's list starts at the
+// number of chosen positions of lower heads plus their windows.
+__global__ void __launch_bounds__(256) adaptive_split_kernel(AdaptArgs a) {
+  const int h = blockIdx.x, l = blockIdx.y;
+  __shared__ int s_lo, s_hi;
+  const int32_t* ch = a.chosen + (size_t)l * a.k_layer;
+  if (threadIdx.x == 0) {
+    if (a.keep_all) {
+      s_lo = h * a.Tv;
+      s_hi = (h + 1) * a.Tv;
+    } else {
+      // first index with ch[i] >= key, for key = h Tv and (h + 1) Tv
+      int lo = 0, hi = a.k_layer;
+      while (lo < hi) {
+        const int m = (lo + hi) >> 1;
+        if (ch[m] < h * a.Tv) lo = m + 1; else hi = m;
+      }
+      s_lo = lo;
+      hi = a.k_layer;
+      while (lo < hi) {
+        const int m = (lo + hi) >> 1;
+        if (ch[m] < (h + 1) * a.Tv) lo = m + 1; else hi = m;
+      }
+      s_hi = lo;
+    }
+  }
+  __syncthreads();
+  const int lo = s_lo, cnt = s_hi - s_lo, off = lo + h * a.W;
+  const size_t base = (size_t)l * a.h_kv * a.n_keep + off;
+  for (int r = threadIdx.x; r < cnt + a.W; r += blockDim.x) {
+    const int pos = r < cnt ? (a.keep_all ? r : ch[lo + r] - h * a.Tv) : a.Tv + (r - cnt);
+    a.idx[base + r] = pos;
+    a.src[base + r] = h * a.N + pos;
+  }
+  if (threadIdx.x == 0) {
+    int32_t* o = a.head_off + (size_t)l * (a.h_kv + 1);
+    o[h] = off;
+    if (h == a.h_kv - 1) o[a.h_kv] = a.h_kv * a.n_keep;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_adaptive_split(const AdaptArgs& a, int n_layers, cudaStream_t s) {
+  adaptive_split_kernel<<<dim3(a.h_kv, n_layers), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 // Scores of every unit and, with do_select, their top-k.
 cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStream_t s) {

@@ -25,7 +25,8 @@ STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED",
 
 EXPORTS = ("ecokv_params_default", "ecokv_check_params", "ecokv_workspace_size", "ecokv_score",
            "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string",
-           "ecokv_evict_noalloc", "ecokv_set_stage_events", "ecokv_workspace_size_host", "ecokv_evict_host")
+           "ecokv_evict_noalloc", "ecokv_set_stage_events", "ecokv_workspace_size_host", "ecokv_evict_host",
+           "ecokv_evict_adaptive")
 
 
 class EcokvError(RuntimeError):
@@ -78,6 +79,8 @@ def lib() -> ctypes.CDLL:
         L.ecokv_workspace_size_host.restype = _sz
         L.ecokv_evict_host.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
         L.ecokv_evict_host.restype = ctypes.c_int
+        L.ecokv_evict_adaptive.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+        L.ecokv_evict_adaptive.restype = ctypes.c_int
         L.ecokv_set_stage_events.argtypes = [ctypes.POINTER(_vp), ctypes.c_int]
         L.ecokv_set_stage_events.restype = ctypes.c_int
         L.ecokv_device_status.argtypes = [_vp, _vp]
@@ -145,6 +148,12 @@ def ecokv_compact(p, dtype, K, V, idx, K_out, V_out, ws=None, ws_bytes=0, stream
 def ecokv_evict(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lam, ws, ws_bytes, stream=None) -> int:
     return lib().ecokv_evict(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx), _ptr(K_out),
                              _ptr(V_out), _ptr(S), _ptr(lam), _ptr(ws), ws_bytes, _stream(stream))
+
+
+def ecokv_evict_adaptive(p, dtype, K, V, Qwin, idx, head_off, K_out, V_out, lam, ws, ws_bytes, stream=None) -> int:
+    return lib().ecokv_evict_adaptive(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx),
+                                      _ptr(head_off), _ptr(K_out), _ptr(V_out), _ptr(lam), _ptr(ws), ws_bytes,
+                                      _stream(stream))
 
 
 def ecokv_workspace_size_host(p, dtype) -> int:
@@ -246,6 +255,22 @@ def evict(p, K, V, Qwin, ws=None, want_scores=False, stream=None):
     _check(ecokv_evict(p, dtype_code(K), K, V, Qwin, idx, Ko, Vo, S, lam, ws, ws.numel(), stream),
            "ecokv_evict")
     return idx, Ko, Vo, S, lam
+
+
+def evict_adaptive(p, K, V, Qwin, ws=None, stream=None):
+    """Run ecokv_evict_adaptive (layer-wide budget); returns (idx [L][h_kv*B],
+    head_off [L][h_kv+1], K_out, V_out [L][h_kv*B][d], lambda)."""
+    import torch
+    ws = alloc_workspace(p, K.device) if ws is None else ws
+    rows = p.h_kv * min(p.budget, p.n)
+    idx = torch.empty(p.n_layers, rows, dtype=torch.int32, device=K.device)
+    off = torch.empty(p.n_layers, p.h_kv + 1, dtype=torch.int32, device=K.device)
+    Ko = torch.empty(p.n_layers, rows, p.d, dtype=K.dtype, device=K.device)
+    Vo = torch.empty_like(Ko)
+    lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32, device=K.device)
+    _check(ecokv_evict_adaptive(p, dtype_code(K), K, V, Qwin, idx, off, Ko, Vo, lam, ws, ws.numel(), stream),
+           "ecokv_evict_adaptive")
+    return idx, off, Ko, Vo, lam
 
 
 def alloc_workspace_host(p, dtype, device="cuda"):
