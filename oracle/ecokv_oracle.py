@@ -41,7 +41,8 @@ listed with its justification in the design notes):
   R5  eps = 1e-6 (a "small constant"), also added to the min-max of S_div.
   R6  S_imp is a sum (not an average) over window rows and group heads; a
       positive per-head scale of S_imp leaves the selection unchanged.
-  R7  No value-norm factor in S_imp (its combination is unspecified).
+  R7  No value-norm factor in S_imp by default (its combination is
+      unspecified); FLAG_VNORM_IMP adds one (R17).
   R8  Scale 1/sqrt(d); window row j sits at position N - W + j and sees keys
       0 .. N - W + j; only the T_v candidates are scored.
   R9  Average pooling, centred, stride 1, zero padding counted in the divisor,
@@ -57,6 +58,9 @@ listed with its justification in the design notes):
   R16 Layer-wide budget (AdaKV): the layer's candidate budget is H_kv (B - W);
       ties across heads go to the lower head, then the lower position; every
       head keeps its whole window.
+  R17 Value-norm importance (FLAG_VNORM_IMP; Sec. 5.2 says S_imp combines the
+      l2 norm of the value vector with the window attention, without the
+      form): S_imp(i) = pooled vote(i) * ||v_i||_2, the pooling first.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -72,6 +76,7 @@ import numpy as np
 
 FLAG_SC_MIXKV_SIGN = 0x1
 FLAG_LAMBDA_OVERRIDE = 0x2
+FLAG_VNORM_IMP = 0x4
 
 NORM_FLOOR = 1e-12
 
@@ -270,10 +275,16 @@ def compact(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
 # --------------------------------------------------------------------------
 # one KV head, then all layers and heads
 # --------------------------------------------------------------------------
-def score_head(K: np.ndarray, Qg: np.ndarray, p: Params) -> dict:
+def value_norms(V: np.ndarray) -> np.ndarray:
+    """||v_i||_2 of every value row (R17)."""
+    return np.sqrt((V * V).sum(axis=1))
+
+
+def score_head(K: np.ndarray, Qg: np.ndarray, p: Params, V: np.ndarray | None = None) -> dict:
     """Every intermediate of the score for one (layer, KV head).
 
-    K: [N, d] float64, Qg: [g, W, d] float64 (the group's window queries).
+    K: [N, d] float64, Qg: [g, W, d] float64 (the group's window queries);
+    V: [N, d] float64, needed with FLAG_VNORM_IMP only.
     """
     n, d = K.shape
     t_v = n - p.window
@@ -285,6 +296,9 @@ def score_head(K: np.ndarray, Qg: np.ndarray, p: Params) -> dict:
     out["lse"] = out["m"] + np.log(np.exp(logits - out["m"][..., None]).sum(-1))
     s_imp_raw = importance_raw(prob, t_v)
     s_imp = avg_pool(s_imp_raw, p.pool_kernel)
+    if p.flags & FLAG_VNORM_IMP:
+        assert V is not None, "FLAG_VNORM_IMP needs the values"
+        s_imp = s_imp * value_norms(V[:t_v])                       # R17
 
     kbar = key_centroid(K)
     d_e_all = euclid_distance(K, kbar)
@@ -333,7 +347,7 @@ def evict_adaptive(K, V, Q, p: Params, layers=None) -> dict:
     g = p.group
     res = {}
     for l in (layers if layers is not None else range(p.n_layers)):
-        heads = [score_head(K[l, h], Q[l, h * g:(h + 1) * g], p) for h in range(p.h_kv)]
+        heads = [score_head(K[l, h], Q[l, h * g:(h + 1) * g], p, V[l, h]) for h in range(p.h_kv)]
         lists = select_adaptive([r["S"] for r in heads], p)
         off = np.concatenate([[0], np.cumsum([len(x) for x in lists])]).astype(np.int64)
         res[l] = {"heads": heads, "idx": np.concatenate(lists), "head_off": off,
@@ -355,7 +369,7 @@ def evict(K, V, Q, p: Params, heads=None) -> dict:
     units = heads if heads is not None else [(l, h) for l in range(p.n_layers) for h in range(p.h_kv)]
     res = {}
     for (l, h) in units:
-        r = score_head(K[l, h], Q[l, h * g:(h + 1) * g], p)
+        r = score_head(K[l, h], Q[l, h * g:(h + 1) * g], p, V[l, h])
         idx = select(r["S"], p)
         r["idx"] = idx
         r["K_out"] = compact(K[l, h], idx)

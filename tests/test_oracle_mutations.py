@@ -127,6 +127,10 @@ def adaptive_no_window(S_heads, p):       # the heads' windows left out
     return [x[x < p.t_v] if p.budget < p.n else x for x in ORIG["select_adaptive"](S_heads, p)]
 
 
+def value_norm_squared(V):               # ||v||^2 instead of ||v||
+    return (V * V).sum(axis=1)
+
+
 MUTANTS = {
     "no_scale": ("window_logits", no_scale),
     "no_causal_mask": ("window_logits", no_causal_mask),
@@ -145,6 +149,7 @@ MUTANTS = {
     "adaptive_budget_counts_window": ("select_adaptive", adaptive_budget_counts_window),
     "adaptive_ties_by_position": ("select_adaptive", adaptive_ties_by_position),
     "adaptive_no_window": ("select_adaptive", adaptive_no_window),
+    "value_norm_squared": ("value_norms", value_norm_squared),
 }
 
 

@@ -412,6 +412,32 @@ def test_evict_adaptive_layout():
     assert np.array_equal(np.concatenate(lists), res["idx"])
 
 
+def test_value_norm_importance_scale_and_selection():
+    # values of one common norm c: S_imp, the rescaled diversity and S all scale
+    # by c (Eq. 7 is homogeneous in S_imp), so the selection is unchanged; a
+    # value row of outsized norm lifts its candidate into the selection
+    r = rng(25)
+    n, d, w, B = 60, 16, 4, 14
+    K, u = aniso(r, n, d)
+    Qg = (4 * u + r.standard_normal((2, w, d)))[:, :, :]
+    V = r.standard_normal((n, d))
+    c = 2.5
+    Vc = c * V / np.linalg.norm(V, axis=1, keepdims=True)
+    base = params(n, d, window=w, budget=B, h_q=2, pool=3)
+    vn = params(n, d, window=w, budget=B, h_q=2, pool=3, flags=O.FLAG_VNORM_IMP)
+    r0 = O.score_head(K, Qg, base)
+    r1 = O.score_head(K, Qg, vn, Vc)
+    assert np.allclose(r1["s_imp"], c * r0["s_imp"], rtol=1e-12, atol=0)
+    assert np.allclose(r1["S"], c * r0["S"], rtol=1e-11, atol=1e-15)
+    assert np.array_equal(O.select(r1["S"], vn), O.select(r0["S"], base))
+    assert np.allclose(O.value_norms(Vc), c)
+    low = int(np.argmin(r0["S"]))
+    Vb = Vc.copy()
+    Vb[low] *= 1e6
+    r2 = O.score_head(K, Qg, vn, Vb)
+    assert low in set(O.select(r2["S"], vn))
+
+
 def test_compact_rows():
     r = rng(18)
     X = r.standard_normal((12, 5))
