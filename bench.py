@@ -49,8 +49,9 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=0,
                     help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--variant", choices=["per-head", "adaptive"], default="per-head",
-                    help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive)")
+    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm"], default="per-head",
+                    help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive); "
+                         "vnorm: importance weighted by the value norms (ECOKV_FLAG_VNORM_IMP)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -300,7 +301,8 @@ def main():
 
     K, V, Q = make_inputs(rank_workload(w, rank), device=dev)
     p = E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
-                      budget=w.budget, pool_kernel=w.pool_kernel)
+                      budget=w.budget, pool_kernel=w.pool_kernel,
+                      flags=E.ECOKV_FLAG_VNORM_IMP if args.variant == "vnorm" else 0)
     ws = E.alloc_workspace(p, dev)
     n_keep = min(w.budget, w.n)
     idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
@@ -376,7 +378,7 @@ def main():
     # Consecutive calls alternate between two streams with their own
     # workspaces, so one call's copy-in overlaps the previous call's kernels.
     e2e = None
-    if args.e2e_steps > 0 and not adaptive:
+    if args.e2e_steps > 0 and args.variant == "per-head":
         hK = K.cpu().pin_memory()
         hV = V.cpu().pin_memory()
         hQ = Q.cpu().pin_memory()
@@ -454,12 +456,15 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
         "data": "synthetic (seeded anisotropic + clustered/temporally correlated keys; no dataset)",
         "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
-                   "variant": "layer-wide budget (ecokv_evict_adaptive)" if adaptive else "per-head budget",
+                   "variant": {"adaptive": "layer-wide budget (ecokv_evict_adaptive)",
+                               "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)"}.get(args.variant,
+                                                                                          "per-head budget"),
                    "evicted_rows_per_s": round(job_rate(world, w.units * max(0, w.n - w.budget), ms_step), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
         # the layer-wide budget adds the layer select (3 digits x 2, count, emit) and the split
-        "gpu_launches": (launches_per_call(w) + (9 if adaptive else 0)) * args.steps, "clocks": clocks,
+        "gpu_launches": (launches_per_call(w) + (9 if adaptive else 0) + (1 if args.variant == "vnorm" else 0))
+        * args.steps, "clocks": clocks,
         "timing": {"headline": f"{args.steps} steps back to back, CUDA events around the region",
                    "stages": f"{args.steps} further steps with per-launch events (launches serialised)",
                    "staged_ms_per_step": round(staged_ms_step, 5)},

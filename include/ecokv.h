@@ -66,6 +66,11 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
 /* variant flags (ecokv_params.flags) */
 #define ECOKV_FLAG_SC_MIXKV_SIGN   0x1u /* s_C = -khat.mu (MixKV, Appendix A) instead of (1 - khat.mu)/2 */
 #define ECOKV_FLAG_LAMBDA_OVERRIDE 0x2u /* use lambda_override for every head (0 = SnapKV importance only) */
+#define ECOKV_FLAG_VNORM_IMP       0x4u /* S_imp(i) = pooled vote(i) * ||v_i||_2 (Sec. 5.2 combines the value
+                                            norm with the window attention; the form is a reading).  Needs V:
+                                            the ecokv_evict* entry points; ecokv_score returns
+                                            ECOKV_ERR_UNSUPPORTED.  Heads of up to 32768 candidates
+                                            (n - window), else ECOKV_ERR_UNSUPPORTED. */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 
 typedef struct {

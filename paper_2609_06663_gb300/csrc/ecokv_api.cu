@@ -48,6 +48,7 @@ Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
   L.chosen = off;  off += align256(U * n_keep * 4);
   L.src = off;     off += align256(U * n_keep * 4);
   L.lsel = off;    off += align256(layer_select_scratch_bytes(p.n_layers, p.h_kv * L.Tv));
+  L.vnorm = off;   off += align256(U * (size_t)L.Tv * 4);
   L.total = off;
   return L;
 }
@@ -248,6 +249,20 @@ static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const
 
 // Scores (and the top-k) of every unit: one cluster per unit when the unit
 // fits eight CTAs, one CTA per unit otherwise.
+// Value-norm importance: reject heads the cluster finalize does not take
+// (before anything is launched), else the norms' launch and their place.
+static ecokv_status vnorm_check(const ecokv_params& p, const Layout& L) {
+  if (!(p.flags & ECOKV_FLAG_VNORM_IMP)) return ECOKV_OK;
+  return cluster_finalize_fits(L.Tv) ? ECOKV_OK : ECOKV_ERR_UNSUPPORTED;
+}
+static ecokv_status vnorm_launch(const ecokv_params& p, ecokv_dtype dt, const Layout& L, const void* V, char* ws,
+                                 FinalArgs& f, cudaStream_t s) {
+  if (!(p.flags & ECOKV_FLAG_VNORM_IMP)) return ECOKV_OK;
+  float* vn = reinterpret_cast<float*>(ws + L.vnorm);
+  f.vnorm = vn;
+  return launch_value_norms(V, dt, L.U, p.n, L.Tv, vn, s) == cudaSuccess ? ECOKV_OK : ECOKV_ERR_CUDA;
+}
+
 static ecokv_status run_finalize(FinalArgs f, int U, bool do_select, cudaStream_t s) {
   if (!do_select) f.idx = nullptr;
   const cudaError_t e = launch_finalize_cluster(f, U, false, s);
@@ -283,7 +298,8 @@ ecokv_status ecokv_check_params(const ecokv_params* p) {
   if (p->pool_kernel < 1 || (p->pool_kernel & 1) == 0) return ECOKV_ERR_INVALID_ARG;
   if (!(p->alpha >= 0.f && p->alpha <= 1.f) || !(p->beta >= 0.f && p->beta <= 1.f)) return ECOKV_ERR_INVALID_ARG;
   if (!(p->eps > 0.f) || !isfinite(p->eps) || !isfinite(p->tau)) return ECOKV_ERR_INVALID_ARG;
-  const uint32_t known = ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_FORCE_SIMT;
+  const uint32_t known =
+      ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_VNORM_IMP | ECOKV_FLAG_FORCE_SIMT;
   if ((p->flags & ~known) != 0u) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_LAMBDA_OVERRIDE) && !isfinite(p->lambda_override)) return ECOKV_ERR_INVALID_ARG;
   if (p->d != kD) return ECOKV_ERR_UNSUPPORTED;
@@ -303,6 +319,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
                          float* lambda, float* dbg, void* ws, size_t ws_bytes, void* stream) {
   ecokv_status st = ecokv_check_params(p);
   if (st != ECOKV_OK) return st;
+  if (p->flags & ECOKV_FLAG_VNORM_IMP) return ECOKV_ERR_UNSUPPORTED;  // needs V: use ecokv_evict
   if (dtype != ECOKV_F32 && dtype != ECOKV_BF16) return ECOKV_ERR_INVALID_ARG;
   if (!K || !Qwin || !aligned16(K) || !aligned16(Qwin)) return ECOKV_ERR_INVALID_ARG;
   if (p->n > p->window && (!S || !aligned16(S))) return ECOKV_ERR_INVALID_ARG;
@@ -382,9 +399,11 @@ ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, cons
   FinalArgs f = final_args(*p, L, w);
   f.S = reinterpret_cast<float*>(w + L.sbuf);
   f.lambda = lambda;
+  if ((st = vnorm_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
+  if ((st = vnorm_launch(*p, dtype, L, V, w, f, s)) != ECOKV_OK) return st;
   stage_event(1, s);
   if (run_finalize(f, L.U, false, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   // 2. one top-h_kv (B - W) per layer over its heads' concatenated scores
@@ -441,9 +460,11 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   f.lambda = lambda;
   f.idx = idx;
   const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, reinterpret_cast<unsigned*>(w + L.status));
+  if ((st = vnorm_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
+  if ((st = vnorm_launch(*p, dtype, L, V, w, f, s)) != ECOKV_OK) return st;
   stage_event(1, s);
   if (run_finalize(f, L.U, true, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   stage_event(2, s);

@@ -51,6 +51,7 @@ struct Layout {
   size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2;
   size_t chosen, src;  // layer-wide budget: chosen positions, gathered rows (U * min(B, N) int32 each)
   size_t lsel;         // layer-wide budget: the layer select's histograms, state and block counts
+  size_t vnorm;        // value-norm importance: ||v_i|| of the candidates, U * Tv floats
   size_t total;
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
@@ -94,6 +95,7 @@ struct FinalArgs {
   float* lambda;     // [U] or null
   float* dbg;        // [U][5][Tv] or null
   int32_t* idx;      // [U][n_keep] or null
+  const float* vnorm;  // [U][Tv] ||v_i|| multiplying the pooled vote (value-norm importance), or null
 };
 
 struct CompactArgs {
@@ -126,6 +128,10 @@ cudaError_t launch_finalize(const FinalArgs& f, int U, bool do_select, cudaStrea
 cudaError_t launch_select(const FinalArgs& f, int U, cudaStream_t s);
 cudaError_t launch_compact(const CompactArgs& a, ecokv_dtype dt, int U, cudaStream_t s);
 cudaError_t launch_adaptive_split(const AdaptArgs& a, int n_layers, cudaStream_t s);
+// ||v_i|| of the Tv candidate rows of every unit: vn[u][i]
+cudaError_t launch_value_norms(const void* V, ecokv_dtype dt, int U, int N, int Tv, float* vn, cudaStream_t s);
+// Whether the cluster finalize takes units of Tv candidates (else one CTA per unit).
+bool cluster_finalize_fits(int Tv);
 // k largest of each layer's T scores, ascending positions (layer_select.cu)
 size_t layer_select_scratch_bytes(int n_layers, int T);
 cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int32_t* chosen, void* scratch,

@@ -67,11 +67,13 @@ struct ClusterSmem {
   // extrema and the counts above / equal to the threshold of every rank.
   unsigned hall[2][Shape<kJ>::kMaxCluster][256];
   float ext_all[Shape<kJ>::kMaxCluster][2];
+  double simp_all[Shape<kJ>::kMaxCluster];  // value-norm importance: every rank's sum of S_imp
   int cnt_all[Shape<kJ>::kMaxCluster][2];
   float red[kCWarps][8];  // per-warp partials
   float edge[32];         // pooling edge values
   float sc[8];            // broadcast scalars
   double dsc[2];          // sums behind the means of S_imp and of S_div
+  double dred[kCWarps];   // per-warp sums of S_imp (value-norm importance)
   unsigned wsum[kCWarps];
   int wscan[kCWarps][2];  // per-warp counts above / equal to the threshold
   int shi[4];
@@ -262,6 +264,31 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     __syncthreads();
     const float mnE = sm.sc[1], denE = sm.sc[2];
     const float invE = __frcp_rn(denE);
+    if (f.vnorm != nullptr) {
+      // value-norm importance: S_imp = pooled vote * ||v||, the norms staged
+      // in coalesced order where the raw votes were; the sum of S_imp (its
+      // mean is no longer a function of the raw-vote sums) goes round the
+      // cluster with the S_div extrema
+      const float* vnu = f.vnorm + (size_t)u * Tv;
+  #pragma unroll 8
+      for (int j = 0; j < kJ; ++j) {
+        const int i = lo + kCThreads * j + tid;
+        if (i < Tv) sm.raw[pad_idx(i - lo + kHalo)] = __ldg(vnu + i);
+      }
+      __syncthreads();
+      double ps = 0.0;
+  #pragma unroll
+      for (int c = 0; c < kJ; ++c)
+        if (c < nv) {
+          const float si = __fmul_rn(__uint_as_float(key[c]), sm.raw[pad_idx(q0 + c)]);
+          key[c] = __float_as_uint(si);
+          ps += (double)si;
+        }
+  #pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
+      if (lane == 0) sm.dred[warp] = ps;
+      __syncthreads();  // also: every norm read before the S_div sweep reuses the buffer
+    }
 
     if (tid == 32) {
       // off the critical path, while the other threads compute S_div:
@@ -366,6 +393,11 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       }
       push_all<kMaxC>(cl, &sm.ext_all[rank][0], a0, C);
       push_all<kMaxC>(cl, &sm.ext_all[rank][1], a1, C);
+      if (f.vnorm != nullptr) {
+        double cs = 0.0;
+        for (int w = 0; w < kCWarps; ++w) cs += sm.dred[w];
+        push_all<kMaxC>(cl, &sm.simp_all[rank], cs, C);
+      }
     }
     cl.sync();
     if (tid == 0) {
@@ -379,7 +411,13 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       const double num = sm.dsc[1] - (double)a0 * (double)Tv;  // Tv * denD * mean(Sbar)
       sm.sc[6] = a0;
       sm.sc[7] = denD;
-      sm.sc[5] = (Tv > 0 && num > 0.0) ? (float)(sm.dsc[0] * (double)denD / ((double)f.pool * num)) : 0.f;
+      double dsc0 = sm.dsc[0];  // kp * Tv * mean(S_imp)
+      if (f.vnorm != nullptr) {
+        double sum_imp = 0.0;
+        for (int r = 0; r < C; ++r) sum_imp += sm.simp_all[r];
+        dsc0 = (double)f.pool * sum_imp;
+      }
+      sm.sc[5] = (Tv > 0 && num > 0.0) ? (float)(dsc0 * (double)denD / ((double)f.pool * num)) : 0.f;
     }
     __syncthreads();
     const float lamf = sm.sc[0], mnD2 = sm.sc[6], denD = sm.sc[7], scale = sm.sc[5];
@@ -628,6 +666,13 @@ cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cud
 }
 
 }  // namespace
+
+bool cluster_finalize_fits(int Tv) {
+  const int t = Tv > 0 ? Tv : 1;
+  const int C16 = (t + Shape<16>::kCap - 1) / Shape<16>::kCap;
+  const int C32 = (t + Shape<32>::kCap - 1) / Shape<32>::kCap;
+  return C16 > 4 ? C32 <= Shape<32>::kMaxCluster : C16 <= Shape<16>::kMaxCluster;
+}
 
 // Scores (and with f.idx the top-k) of every unit, or with select_only the
 // top-k of the scores in f.S; one cluster per unit; cudaErrorNotSupported

@@ -82,7 +82,59 @@ __global__ void __launch_bounds__(256) adaptive_split_kernel(AdaptArgs a) {
   }
 }
 
+// ||v_i|| for the candidate rows: 16-byte vectors, the lanes of a row summing
+// their squares in fp32 and combining by shuffles (a streaming read of V).
+template <typename T>
+__global__ void __launch_bounds__(256) value_norm_kernel(const T* V, float* vn, int N, int Tv) {
+  constexpr int kVpr = kD * sizeof(T) / 16;  // 16-byte vectors per row: 16 (bf16) or 32 (fp32)
+  constexpr int kRows = 32 / kVpr;           // rows a warp takes per step
+  const int u = blockIdx.y, lane = threadIdx.x & 31;
+  const int r_lane = lane / kVpr, v = lane % kVpr;
+  const uint4* Vu = reinterpret_cast<const uint4*>(V) + (size_t)u * N * kVpr;
+  const int warps = gridDim.x * (blockDim.x >> 5), w = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int step = warps * kRows;
+  for (int r0 = w * kRows; r0 < Tv; r0 += 4 * step) {
+    uint4 q[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int r = r0 + j * step + r_lane;
+      q[j] = r < Tv ? __ldcs(Vu + (size_t)r * kVpr + v) : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int r = r0 + j * step + r_lane;
+      float acc = 0.f;
+      if constexpr (sizeof(T) == 2) {
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q[j]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(h[e]);
+          acc = fmaf(f.x, f.x, acc);
+          acc = fmaf(f.y, f.y, acc);
+        }
+      } else {
+        const float* f = reinterpret_cast<const float*>(&q[j]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc = fmaf(f[e], f[e], acc);
+      }
+#pragma unroll
+      for (int o = kVpr / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      if (v == 0 && r < Tv) vn[(size_t)u * Tv + r] = sqrtf(acc);
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_value_norms(const void* V, ecokv_dtype dt, int U, int N, int Tv, float* vn, cudaStream_t s) {
+  if (U <= 0 || Tv <= 0) return cudaSuccess;
+  const dim3 grid((unsigned)((Tv + 255) / 256 < 64 ? (Tv + 255) / 256 : 64), U);
+  if (dt == ECOKV_F32)
+    value_norm_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(V), vn, N, Tv);
+  else
+    value_norm_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(V), vn, N, Tv);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_adaptive_split(const AdaptArgs& a, int n_layers, cudaStream_t s) {
   adaptive_split_kernel<<<dim3(a.h_kv, n_layers), 256, 0, s>>>(a);
