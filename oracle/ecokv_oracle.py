@@ -21,7 +21,9 @@ Sec. 5.1-5.2 Eq. 1-7, Appendix A "SnapKV" and "MixKV", Algorithm 1):
      (Sec. 3), and the gather of the retained K/V rows;
   7. (variant, AdaKV's layer-wide budget, Appendix A) one top-H_kv (B - W)
      over the concatenated scores of a layer's heads instead of one top-(B - W)
-     per head.
+     per head;
+  8. (variant, PyramidKV's per-layer budgets, Appendix A) budget b^l for the
+     heads of layer l.
 
 Readings of passages that are silent, ambiguous or garbled (each one is also
 listed with its justification in the design notes):
@@ -61,6 +63,9 @@ listed with its justification in the design notes):
   R17 Value-norm importance (FLAG_VNORM_IMP; Sec. 5.2 says S_imp combines the
       l2 norm of the value vector with the window attention, without the
       form): S_imp(i) = pooled vote(i) * ||v_i||_2, the pooling first.
+  R18 Per-layer budgets (PyramidKV, Appendix A): the total is the uniform
+      budget's, m B; the real-valued schedule is rounded half up and raised to
+      at least W; a layer budget >= N keeps the layer whole.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -336,6 +341,34 @@ def to_f64(x) -> np.ndarray:
     if hasattr(x, "detach"):                      # torch tensor, without importing torch
         x = x.detach().cpu().double().numpy()
     return np.asarray(x, dtype=np.float64)
+
+
+def pyramid_budgets_real(m: int, b_total: float, beta: float) -> list:
+    """PyramidKV's per-layer budgets (Appendix A): b^{m-1} = b_total / (beta m),
+    b^0 = 2 b_total / m - b^{m-1}, and b^l linear between them."""
+    if m == 1:
+        return [float(b_total)]
+    b_last = b_total / (beta * m)
+    b_first = 2.0 * b_total / m - b_last
+    return [b_first - (b_first - b_last) / (m - 1) * l for l in range(m)]
+
+
+def pyramid_budgets(m: int, budget: int, beta: float, window: int) -> list:
+    """Integer per-layer budgets (reading R18): the uniform budget's total
+    m B spread by pyramid_budgets_real, each rounded half up and raised to at
+    least the window."""
+    return [max(window, int(np.floor(x + 0.5))) for x in pyramid_budgets_real(m, m * budget, beta)]
+
+
+def evict_layered(K, V, Q, p: Params, budgets: list, heads=None) -> dict:
+    """The pass with budget budgets[l] for every head of layer l (PyramidKV
+    schedule); otherwise as evict."""
+    res = {}
+    units = heads if heads is not None else [(l, h) for l in range(p.n_layers) for h in range(p.h_kv)]
+    for l in sorted({l for l, _ in units}):
+        pl = Params(**{**p.__dict__, "budget": int(budgets[l])})
+        res.update(evict(K, V, Q, pl, heads=[(ll, h) for ll, h in units if ll == l]))
+    return res
 
 
 def evict_adaptive(K, V, Q, p: Params, layers=None) -> dict:

@@ -131,6 +131,22 @@ def value_norm_squared(V):               # ||v||^2 instead of ||v||
     return (V * V).sum(axis=1)
 
 
+def pyramid_top_without_m(m, b_total, beta):    # b^{m-1} = b_total / beta
+    if m == 1:
+        return [float(b_total)]
+    b_last = b_total / beta
+    b_first = 2.0 * b_total / m - b_last
+    return [b_first - (b_first - b_last) / (m - 1) * l for l in range(m)]
+
+
+def pyramid_step_over_m(m, b_total, beta):      # slope divided by m, not m - 1
+    if m == 1:
+        return [float(b_total)]
+    b_last = b_total / (beta * m)
+    b_first = 2.0 * b_total / m - b_last
+    return [b_first - (b_first - b_last) / m * l for l in range(m)]
+
+
 MUTANTS = {
     "no_scale": ("window_logits", no_scale),
     "no_causal_mask": ("window_logits", no_causal_mask),
@@ -150,6 +166,8 @@ MUTANTS = {
     "adaptive_ties_by_position": ("select_adaptive", adaptive_ties_by_position),
     "adaptive_no_window": ("select_adaptive", adaptive_no_window),
     "value_norm_squared": ("value_norms", value_norm_squared),
+    "pyramid_top_without_m": ("pyramid_budgets_real", pyramid_top_without_m),
+    "pyramid_step_over_m": ("pyramid_budgets_real", pyramid_step_over_m),
 }
 
 

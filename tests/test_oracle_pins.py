@@ -438,6 +438,26 @@ def test_value_norm_importance_scale_and_selection():
     assert low in set(O.select(r2["S"], vn))
 
 
+@pytest.mark.parametrize("m,b_total,beta", [(28, 28 * 3277, 20.0), (32, 32 * 205, 20.0), (5, 500, 3.0),
+                                             (2, 64, 1.5)])
+def test_pyramid_schedule_closed_forms(m, b_total, beta):
+    b = O.pyramid_budgets_real(m, b_total, beta)
+    assert math.isclose(sum(b), b_total, rel_tol=1e-12)               # the total is kept
+    assert math.isclose(b[-1], b_total / (beta * m), rel_tol=1e-12)   # the top layer
+    assert math.isclose(b[0] + b[-1], 2 * b_total / m, rel_tol=1e-12)
+    steps = np.diff(b)
+    assert np.allclose(steps, steps[0], rtol=1e-9) and steps[0] <= 0  # linear, decreasing for beta >= 1
+
+
+def test_pyramid_uniform_when_beta_is_one_and_integer_reading():
+    assert O.pyramid_budgets_real(6, 600, 1.0) == pytest.approx([100.0] * 6)
+    assert O.pyramid_budgets(6, 100, 1.0, 4) == [100] * 6
+    got = O.pyramid_budgets(28, 3277, 20.0, 8)
+    real = O.pyramid_budgets_real(28, 28 * 3277, 20.0)
+    assert all(abs(g - r) <= 0.5 for g, r in zip(got, real))
+    assert O.pyramid_budgets(4, 10, 100.0, 8)[-1] == 8                # raised to the window
+
+
 def test_compact_rows():
     r = rng(18)
     X = r.standard_normal((12, 5))
