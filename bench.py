@@ -49,9 +49,10 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=0,
                     help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm"], default="per-head",
+    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm", "pyramid"], default="per-head",
                     help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive); "
-                         "vnorm: importance weighted by the value norms (ECOKV_FLAG_VNORM_IMP)")
+                         "vnorm: importance weighted by the value norms (ECOKV_FLAG_VNORM_IMP); "
+                         "pyramid: PyramidKV per-layer budgets, beta 20 (ecokv_evict_layered)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -300,11 +301,12 @@ def main():
     from paper_2609_06663_gb300.workloads import make_inputs
 
     K, V, Q = make_inputs(rank_workload(w, rank), device=dev)
+    budgets = E.pyramid_budgets(w.n_layers, w.budget, w.window, 20.0) if args.variant == "pyramid" else None
     p = E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
-                      budget=w.budget, pool_kernel=w.pool_kernel,
+                      budget=max(budgets) if budgets else w.budget, pool_kernel=w.pool_kernel,
                       flags=E.ECOKV_FLAG_VNORM_IMP if args.variant == "vnorm" else 0)
     ws = E.alloc_workspace(p, dev)
-    n_keep = min(w.budget, w.n)
+    n_keep = min(p.budget, w.n)
     idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
     Ko = torch.empty(w.n_layers, w.h_kv, n_keep, w.d, dtype=K.dtype, device=dev)
     Vo = torch.empty_like(Ko)
@@ -320,9 +322,14 @@ def main():
         Ko_a = torch.empty(w.n_layers, rows, w.d, dtype=K.dtype, device=dev)
         Vo_a = torch.empty_like(Ko_a)
 
+    lb_host = torch.tensor(budgets, dtype=torch.int32) if budgets else None
+
     def step():
         if adaptive:
             code = E.ecokv_evict_adaptive(p, dt, K, V, Q, idx_a, off_a, Ko_a, Vo_a, lam, ws, ws.numel(), stream)
+        elif budgets:
+            code = E.ecokv_evict_layered(p, dt, K, V, Q, lb_host.data_ptr(), idx, Ko, Vo, None, lam, ws, ws.numel(),
+                                         stream)
         else:
             code = E.ecokv_evict(p, dt, K, V, Q, idx, Ko, Vo, None, lam, ws, ws.numel(), stream)
         if code:
@@ -457,8 +464,9 @@ def main():
         "data": "synthetic (seeded anisotropic + clustered/temporally correlated keys; no dataset)",
         "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
                    "variant": {"adaptive": "layer-wide budget (ecokv_evict_adaptive)",
-                               "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)"}.get(args.variant,
-                                                                                          "per-head budget"),
+                               "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)",
+                               "pyramid": f"per-layer budgets, PyramidKV beta 20: {budgets}"}.get(
+                                   args.variant, "per-head budget"),
                    "evicted_rows_per_s": round(job_rate(world, w.units * max(0, w.n - w.budget), ms_step), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,

@@ -137,6 +137,27 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
                          const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S,
                          float* lambda, void* ws, size_t ws_bytes, void* stream);
 
+/* The whole pass with a budget per layer (PyramidKV, Appendix A): the heads
+ * of layer l keep layer_budget[l] rows (window included; layer_budget[l] >= n
+ * keeps the layer whole) instead of p->budget.
+ *   layer_budget : host array of n_layers entries, each in [window, p->budget];
+ *                  ecokv_pyramid_budgets gives PyramidKV's schedule.
+ *   idx, K_out, V_out : as for ecokv_evict, with p->budget the per-head stride:
+ *                  head (l, h) fills its first min(layer_budget[l], n) slots;
+ *                  the idx slots after them hold -1 and those K_out / V_out
+ *                  rows are not written.
+ *   Everything else as for ecokv_evict.  n_layers <= 256 (else
+ *   ECOKV_ERR_UNSUPPORTED). */
+ecokv_status ecokv_evict_layered(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                                 const void* Qwin, const int32_t* layer_budget, int32_t* idx, void* K_out,
+                                 void* V_out, float* S, float* lambda, void* ws, size_t ws_bytes, void* stream);
+
+/* PyramidKV's per-layer budgets (Appendix A) for n_layers layers keeping
+ * n_layers * budget rows per head in all: b^{m-1} = total / (beta m),
+ * b^0 = 2 total / m - b^{m-1}, linear in between, each rounded half up and at
+ * least `window`.  beta > 0 shapes the pyramid (1 = uniform).  Host only. */
+ecokv_status ecokv_pyramid_budgets(int32_t n_layers, int32_t budget, int32_t window, float beta, int32_t* out);
+
 /* The whole pass with a layer-wide budget (AdaKV, Appendix A): instead of
  * each head keeping its own top-(B - W), the heads of a layer share one
  * budget of h_kv (B - W) candidates, taken as one top-K over their

@@ -157,6 +157,7 @@ static FinalArgs final_args(const ecokv_params& p, const Layout& L, char* ws) {
   f.lambda_override = p.lambda_override;
   f.flags = p.flags;
   f.n_keep = p.budget < p.n ? p.budget : p.n;
+  f.h_kv = p.h_kv;
   if (ws != nullptr) {
     f.p2part = reinterpret_cast<const float*>(ws + L.p2part);
     f.ustat = reinterpret_cast<const float*>(ws + L.ustat);
@@ -178,6 +179,7 @@ static CompactArgs compact_args(const ecokv_params& p, const void* K, const void
   c.N = p.n;
   c.n_keep = p.budget < p.n ? p.budget : p.n;
   c.status = status;
+  c.h_kv = p.h_kv;
   return c;
 }
 
@@ -438,9 +440,9 @@ ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, cons
   return ECOKV_OK;
 }
 
-ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V, const void* Qwin,
-                         int32_t* idx, void* K_out, void* V_out, float* S, float* lambda, void* ws,
-                         size_t ws_bytes, void* stream) {
+static ecokv_status evict_impl(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                               const void* Qwin, int32_t* idx, void* K_out, void* V_out, float* S, float* lambda,
+                               void* ws, size_t ws_bytes, void* stream, const int32_t* layer_budget) {
   ecokv_status st = ecokv_check_params(p);
   if (st != ECOKV_OK) return st;
   if (dtype != ECOKV_F32 && dtype != ECOKV_BF16) return ECOKV_ERR_INVALID_ARG;
@@ -459,7 +461,14 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);
   f.lambda = lambda;
   f.idx = idx;
-  const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, reinterpret_cast<unsigned*>(w + L.status));
+  CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, reinterpret_cast<unsigned*>(w + L.status));
+  if (layer_budget != nullptr) {
+    f.n_lb = c.n_lb = p->n_layers;
+    for (int l = 0; l < p->n_layers; ++l) {
+      f.lb[l] = layer_budget[l];
+      c.keep[l] = layer_budget[l] < p->n ? layer_budget[l] : p->n;
+    }
+  }
   if ((st = vnorm_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
@@ -470,6 +479,44 @@ ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K
   stage_event(2, s);
   if (launch_compact(c, dtype, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   stage_event(3, s);
+  return ECOKV_OK;
+}
+
+ecokv_status ecokv_evict(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V, const void* Qwin,
+                         int32_t* idx, void* K_out, void* V_out, float* S, float* lambda, void* ws,
+                         size_t ws_bytes, void* stream) {
+  return evict_impl(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lambda, ws, ws_bytes, stream, nullptr);
+}
+
+ecokv_status ecokv_evict_layered(const ecokv_params* p, ecokv_dtype dtype, const void* K, const void* V,
+                                 const void* Qwin, const int32_t* layer_budget, int32_t* idx, void* K_out,
+                                 void* V_out, float* S, float* lambda, void* ws, size_t ws_bytes, void* stream) {
+  ecokv_status st = ecokv_check_params(p);
+  if (st != ECOKV_OK) return st;
+  if (layer_budget == nullptr) return ECOKV_ERR_INVALID_ARG;
+  if (p->n_layers > kMaxLayerBudgets) return ECOKV_ERR_UNSUPPORTED;
+  for (int l = 0; l < p->n_layers; ++l)
+    if (layer_budget[l] < p->window || layer_budget[l] > p->budget) return ECOKV_ERR_INVALID_ARG;
+  return evict_impl(p, dtype, K, V, Qwin, idx, K_out, V_out, S, lambda, ws, ws_bytes, stream, layer_budget);
+}
+
+ecokv_status ecokv_pyramid_budgets(int32_t n_layers, int32_t budget, int32_t window, float beta, int32_t* out) {
+  if (n_layers < 1 || budget < window || window < 1 || !(beta > 0.f) || !isfinite(beta) || out == nullptr)
+    return ECOKV_ERR_INVALID_ARG;
+  // PyramidKV (Appendix A): b^{m-1} = b_total / (beta m), b^0 = 2 b_total / m
+  // - b^{m-1}, linear between; b_total = m B; rounded half up, at least W
+  const double m = (double)n_layers, total = m * (double)budget, b = (double)beta;
+  if (n_layers == 1) {
+    out[0] = budget;
+    return ECOKV_OK;
+  }
+  const double b_last = total / (b * m);
+  const double b_first = 2.0 * total / m - b_last;
+  for (int l = 0; l < n_layers; ++l) {
+    const double x = b_first - (b_first - b_last) / (m - 1.0) * (double)l;
+    const double r = floor(x + 0.5);
+    out[l] = r < (double)window ? window : (r > 2147483647.0 ? 2147483647 : (int32_t)r);
+  }
   return ECOKV_OK;
 }
 

@@ -80,6 +80,8 @@ struct ScoreArgs {
   float* cosv;
 };
 
+constexpr int kMaxLayerBudgets = 256;  // layers a per-layer budget schedule may have
+
 struct FinalArgs {
   int N, W, Tv, nchunks, budget, pool, ustat_stride;
   float alpha, beta, tau, eps, lambda_override;
@@ -96,7 +98,14 @@ struct FinalArgs {
   float* dbg;        // [U][5][Tv] or null
   int32_t* idx;      // [U][n_keep] or null
   const float* vnorm;  // [U][Tv] ||v_i|| multiplying the pooled vote (value-norm importance), or null
+  // per-layer budgets (PyramidKV schedule): with n_lb > 0 the heads of layer
+  // l keep lb[l] rows (window included) in slots of stride n_keep
+  int h_kv, n_lb;
+  int lb[kMaxLayerBudgets];
 };
+
+// The budget of unit u (layer u / h_kv).
+__host__ __device__ inline int unit_budget(const FinalArgs& f, int u) { return f.n_lb ? f.lb[u / f.h_kv] : f.budget; }
 
 struct CompactArgs {
   const void* K;
@@ -106,6 +115,9 @@ struct CompactArgs {
   void* V_out;
   int N, n_keep;
   unsigned* status;  // may be null
+  // per-layer budgets: unit u copies keep[u / h_kv] rows (of stride n_keep)
+  int h_kv, n_lb;
+  int keep[kMaxLayerBudgets];
 };
 
 // Layer-wide budget (AdaKV): the split of each layer's chosen positions into

@@ -121,8 +121,9 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   const int c0 = lo + kJ * tid;     // first candidate of this thread
   const int q0 = kJ * tid + kHalo;  // staged position of candidate c0
   const int nv = max(0, min(kJ, Tv - c0));  // of this thread's candidates, those below Tv
-  const bool keep_all = f.budget >= f.N;
-  const int k = keep_all ? 0 : f.budget - f.W;
+  const int budget = unit_budget(f, u);
+  const bool keep_all = budget >= f.N;
+  const int k = keep_all ? 0 : budget - f.W;
   const bool mix = (f.flags & ECOKV_FLAG_SC_MIXKV_SIGN) != 0;
   const int hpool = f.pool >> 1;
   const bool pool_smem = hpool <= kHalo;
@@ -625,6 +626,8 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     } else if (rank == C - 1) {
       for (int j = tid; j < f.W; j += kCThreads) out[k + j] = Tv + j;
     }
+    if (rank == C - 1)  // slots past this unit's budget (per-layer budgets) hold -1
+      for (int r = (keep_all ? f.N : budget) + tid; r < f.n_keep; r += kCThreads) out[r] = -1;
   }
   // No CTA touches a peer's shared memory after the last cluster barrier it
   // passed (every exchange is a store made before that barrier), so the

@@ -313,11 +313,14 @@ __device__ void topk_ascending(const float* S, int Tv, int k, int32_t* out, unsi
 template <class Sync>
 __device__ void select_unit(const FinalArgs& a, int u, const float* S, unsigned* hist, int* shi, int tid, int nt) {
   int32_t* out = a.idx + (size_t)u * a.n_keep;
-  if (a.budget >= a.N) {
+  const int budget = unit_budget(a, u);
+  // slots past this unit's budget (per-layer budgets) hold -1
+  for (int r = (budget < a.N ? budget : a.N) + tid; r < a.n_keep; r += nt) out[r] = -1;
+  if (budget >= a.N) {
     for (int r = tid; r < a.N; r += nt) out[r] = r;
     return;
   }
-  const int k = a.budget - a.W;
+  const int k = budget - a.W;
   topk_ascending<Sync>(S, a.Tv, k, out, hist, shi, tid, nt);
   for (int j = tid; j < a.W; j += nt) out[k + j] = a.Tv + j;
 }
@@ -332,7 +335,7 @@ __device__ void gather_rows(const CompactArgs& a, int u, int r0, int r1, int tid
   uint4* Ko = reinterpret_cast<uint4*>(a.K_out) + (size_t)u * a.n_keep * vpr;
   uint4* Vo = reinterpret_cast<uint4*>(a.V_out) + (size_t)u * a.n_keep * vpr;
   const int32_t* idx = a.idx + (size_t)u * a.n_keep;
-  r1 = min(r1, a.n_keep);
+  r1 = min(r1, a.n_lb ? a.keep[u / a.h_kv] : a.n_keep);
   const int total = (r1 - r0) * vpr;
   for (int e0 = tid; e0 < total; e0 += 4 * nt) {
     uint4 kv[4], vv[4];

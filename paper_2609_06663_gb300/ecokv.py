@@ -27,7 +27,7 @@ STATUS = {0: "ECOKV_OK", 1: "ECOKV_ERR_INVALID_ARG", 2: "ECOKV_ERR_UNSUPPORTED",
 EXPORTS = ("ecokv_params_default", "ecokv_check_params", "ecokv_workspace_size", "ecokv_score",
            "ecokv_select", "ecokv_compact", "ecokv_evict", "ecokv_device_status", "ecokv_status_string",
            "ecokv_evict_noalloc", "ecokv_set_stage_events", "ecokv_workspace_size_host", "ecokv_evict_host",
-           "ecokv_evict_adaptive")
+           "ecokv_evict_adaptive", "ecokv_evict_layered", "ecokv_pyramid_budgets")
 
 
 class EcokvError(RuntimeError):
@@ -82,6 +82,11 @@ def lib() -> ctypes.CDLL:
         L.ecokv_evict_host.restype = ctypes.c_int
         L.ecokv_evict_adaptive.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
         L.ecokv_evict_adaptive.restype = ctypes.c_int
+        L.ecokv_evict_layered.argtypes = [_P, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                          _vp]
+        L.ecokv_evict_layered.restype = ctypes.c_int
+        L.ecokv_pyramid_budgets.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_float, _vp]
+        L.ecokv_pyramid_budgets.restype = ctypes.c_int
         L.ecokv_set_stage_events.argtypes = [ctypes.POINTER(_vp), ctypes.c_int]
         L.ecokv_set_stage_events.restype = ctypes.c_int
         L.ecokv_device_status.argtypes = [_vp, _vp]
@@ -155,6 +160,20 @@ def ecokv_evict_adaptive(p, dtype, K, V, Qwin, idx, head_off, K_out, V_out, lam,
     return lib().ecokv_evict_adaptive(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(idx),
                                       _ptr(head_off), _ptr(K_out), _ptr(V_out), _ptr(lam), _ptr(ws), ws_bytes,
                                       _stream(stream))
+
+
+def ecokv_evict_layered(p, dtype, K, V, Qwin, layer_budget, idx, K_out, V_out, S, lam, ws, ws_bytes,
+                        stream=None) -> int:
+    return lib().ecokv_evict_layered(ctypes.byref(p), dtype, _ptr(K), _ptr(V), _ptr(Qwin), _ptr(layer_budget),
+                                     _ptr(idx), _ptr(K_out), _ptr(V_out), _ptr(S), _ptr(lam), _ptr(ws), ws_bytes,
+                                     _stream(stream))
+
+
+def pyramid_budgets(n_layers: int, budget: int, window: int, beta: float) -> list:
+    """PyramidKV's per-layer budgets from the library (host computation)."""
+    out = (ctypes.c_int32 * n_layers)()
+    _check(lib().ecokv_pyramid_budgets(n_layers, budget, window, beta, ctypes.addressof(out)), "ecokv_pyramid_budgets")
+    return list(out)
 
 
 def ecokv_workspace_size_host(p, dtype) -> int:
@@ -272,6 +291,24 @@ def evict_adaptive(p, K, V, Qwin, ws=None, stream=None):
     _check(ecokv_evict_adaptive(p, dtype_code(K), K, V, Qwin, idx, off, Ko, Vo, lam, ws, ws.numel(), stream),
            "ecokv_evict_adaptive")
     return idx, off, Ko, Vo, lam
+
+
+def evict_layered(p, K, V, Qwin, budgets, ws=None, want_scores=False, stream=None):
+    """Run ecokv_evict_layered with budgets[l] for layer l (p.budget is the
+    per-head stride, at least max(budgets)); returns as evict()."""
+    import torch
+    ws = alloc_workspace(p, K.device) if ws is None else ws
+    n_keep = min(p.budget, p.n)
+    lb = torch.tensor(list(budgets), dtype=torch.int32)
+    idx = torch.empty(p.n_layers, p.h_kv, n_keep, dtype=torch.int32, device=K.device)
+    Ko = torch.zeros(p.n_layers, p.h_kv, n_keep, p.d, dtype=K.dtype, device=K.device)
+    Vo = torch.zeros_like(Ko)
+    S = torch.empty(p.n_layers, p.h_kv, p.n - p.window, dtype=torch.float32, device=K.device) \
+        if want_scores else None
+    lam = torch.empty(p.n_layers, p.h_kv, dtype=torch.float32, device=K.device)
+    _check(ecokv_evict_layered(p, dtype_code(K), K, V, Qwin, lb.data_ptr(), idx, Ko, Vo, S, lam, ws, ws.numel(),
+                               stream), "ecokv_evict_layered")
+    return idx, Ko, Vo, S, lam
 
 
 def alloc_workspace_host(p, dtype, device="cuda"):

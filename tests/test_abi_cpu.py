@@ -95,6 +95,31 @@ def test_entry_points_reject_bad_arguments_before_launch(lib):
     assert E.ecokv_evict(p, 1, fake, fake, fake, fake, fake, fake, None, None, fake, ws_need) == 2
 
 
+@pytest.mark.parametrize("m,B,W,beta", [(28, 3277, 8, 20.0), (32, 205, 8, 20.0), (28, 1024, 4, 5.0), (1, 50, 4, 20.0),
+                                       (4, 10, 8, 100.0), (6, 100, 4, 1.0)])
+def test_pyramid_budgets_match_the_oracle(lib, m, B, W, beta):
+    from oracle import ecokv_oracle as O
+    import numpy as np
+    beta32 = float(np.float32(beta))
+    assert E.pyramid_budgets(m, B, W, beta) == O.pyramid_budgets(m, B, beta32, W)
+
+
+def test_pyramid_budgets_and_layered_entry_reject_bad_arguments(lib):
+    import ctypes
+    out = (ctypes.c_int32 * 4)()
+    assert lib.ecokv_pyramid_budgets(4, 3, 8, 20.0, ctypes.addressof(out)) == 1   # budget below the window
+    assert lib.ecokv_pyramid_budgets(4, 100, 8, 0.0, ctypes.addressof(out)) == 1  # beta must be > 0
+    p = good()
+    fake = 1 << 20
+    ws = E.ecokv_workspace_size(p)
+    lb = (ctypes.c_int32 * 2)(600, 100)                                            # above p.budget = 512
+    assert E.ecokv_evict_layered(p, 1, fake, fake, fake, ctypes.addressof(lb), fake, fake, fake, None, None, fake,
+                                 ws) == 1
+    lb = (ctypes.c_int32 * 2)(2, 100)                                              # below the window
+    assert E.ecokv_evict_layered(p, 1, fake, fake, fake, ctypes.addressof(lb), fake, fake, fake, None, None, fake,
+                                 ws) == 1
+
+
 def test_status_strings(lib):
     for c in range(7):
         assert E.ecokv_status_string(c)
