@@ -49,10 +49,11 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=0,
                     help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm", "pyramid"], default="per-head",
+    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm", "pyramid", "centroid-nonwin"], default="per-head",
                     help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive); "
                          "vnorm: importance weighted by the value norms (ECOKV_FLAG_VNORM_IMP); "
-                         "pyramid: PyramidKV per-layer budgets, beta 20 (ecokv_evict_layered)")
+                         "pyramid: PyramidKV per-layer budgets, beta 20 (ecokv_evict_layered); "
+                         "centroid-nonwin: the centroid over the candidates only (ECOKV_FLAG_CENTROID_NONWIN)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -304,7 +305,8 @@ def main():
     budgets = E.pyramid_budgets(w.n_layers, w.budget, w.window, 20.0) if args.variant == "pyramid" else None
     p = E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
                       budget=max(budgets) if budgets else w.budget, pool_kernel=w.pool_kernel,
-                      flags=E.ECOKV_FLAG_VNORM_IMP if args.variant == "vnorm" else 0)
+                      flags={"vnorm": E.ECOKV_FLAG_VNORM_IMP,
+                             "centroid-nonwin": E.ECOKV_FLAG_CENTROID_NONWIN}.get(args.variant, 0))
     ws = E.alloc_workspace(p, dev)
     n_keep = min(p.budget, w.n)
     idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
@@ -465,7 +467,8 @@ def main():
         "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
                    "variant": {"adaptive": "layer-wide budget (ecokv_evict_adaptive)",
                                "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)",
-                               "pyramid": f"per-layer budgets, PyramidKV beta 20: {budgets}"}.get(
+                               "pyramid": f"per-layer budgets, PyramidKV beta 20: {budgets}",
+                               "centroid-nonwin": "non-window centroid (ECOKV_FLAG_CENTROID_NONWIN)"}.get(
                                    args.variant, "per-head budget"),
                    "evicted_rows_per_s": round(job_rate(world, w.units * max(0, w.n - w.budget), ms_step), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},

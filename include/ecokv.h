@@ -71,6 +71,9 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
                                             the ecokv_evict* entry points; ecokv_score returns
                                             ECOKV_ERR_UNSUPPORTED.  Heads of up to 32768 candidates
                                             (n - window), else ECOKV_ERR_UNSUPPORTED. */
+#define ECOKV_FLAG_CENTROID_NONWIN 0x8u /* the centroid kbar of Eq. 1 over the n - window candidates only
+                                            (Appendix B's alternative to Algorithm 1 step 5; all keys when
+                                            n = window); d_E, D_E, mu and r_C otherwise as by default */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 
 typedef struct {

@@ -66,6 +66,10 @@ listed with its justification in the design notes):
   R18 Per-layer budgets (PyramidKV, Appendix A): the total is the uniform
       budget's, m B; the real-valued schedule is rounded half up and raised to
       at least W; a layer budget >= N keeps the layer whole.
+  R19 Non-window centroid (FLAG_CENTROID_NONWIN; Appendix B's alternative to
+      Algorithm 1 step 5): kbar over the T_v candidates (all N keys when
+      T_v = 0); d_E of every key to that centroid, D_E still over all N (Eq.
+      4); mu and r_C unchanged.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -82,6 +86,7 @@ import numpy as np
 FLAG_SC_MIXKV_SIGN = 0x1
 FLAG_LAMBDA_OVERRIDE = 0x2
 FLAG_VNORM_IMP = 0x4
+FLAG_CENTROID_NONWIN = 0x8
 
 NORM_FLOOR = 1e-12
 
@@ -305,7 +310,7 @@ def score_head(K: np.ndarray, Qg: np.ndarray, p: Params, V: np.ndarray | None = 
         assert V is not None, "FLAG_VNORM_IMP needs the values"
         s_imp = s_imp * value_norms(V[:t_v])                       # R17
 
-    kbar = key_centroid(K)
+    kbar = key_centroid(K[:t_v] if (p.flags & FLAG_CENTROID_NONWIN) and t_v > 0 else K)   # R4, R19
     d_e_all = euclid_distance(K, kbar)
     D_E = d_e_all.mean()                                          # Eq. 4, all T keys
     r_E = euclid_redundancy(D_E, p.tau_eff)

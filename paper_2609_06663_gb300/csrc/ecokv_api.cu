@@ -116,6 +116,12 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
   return x < lo ? lo : (x > hi ? hi : x);
 }
 
+// Keys forming the centroid of Eq. 1: all N, or with the non-window centroid
+// the Tv candidates (all N when there are none).
+static int kbar_count(const ecokv_params& p, const Layout& L) {
+  return (p.flags & ECOKV_FLAG_CENTROID_NONWIN) && L.Tv > 0 ? L.Tv : L.N;
+}
+
 static ScoreArgs score_args(const ecokv_params& p, const Layout& L, const void* K, const void* Q, char* ws) {
   ScoreArgs a{};
   a.K = K;
@@ -127,6 +133,7 @@ static ScoreArgs score_args(const ecokv_params& p, const Layout& L, const void* 
   a.h_kv = p.h_kv;
   a.h_q = p.h_q;
   a.Tv = L.Tv;
+  a.kbar_n = kbar_count(p, L);
   a.nchunks = L.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;
@@ -200,6 +207,7 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.h_kv = p.h_kv;
   a.h_q = p.h_q;
   a.Tv = L.Tv;
+  a.kbar_n = kbar_count(p, L);
   a.q_rows = p.n_layers * p.h_q * p.window;
   a.tiles_per_chunk = tiles;
   a.nchunks = L.nchunks;
@@ -301,7 +309,8 @@ ecokv_status ecokv_check_params(const ecokv_params* p) {
   if (!(p->alpha >= 0.f && p->alpha <= 1.f) || !(p->beta >= 0.f && p->beta <= 1.f)) return ECOKV_ERR_INVALID_ARG;
   if (!(p->eps > 0.f) || !isfinite(p->eps) || !isfinite(p->tau)) return ECOKV_ERR_INVALID_ARG;
   const uint32_t known =
-      ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_VNORM_IMP | ECOKV_FLAG_FORCE_SIMT;
+      ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_VNORM_IMP | ECOKV_FLAG_CENTROID_NONWIN |
+      ECOKV_FLAG_FORCE_SIMT;
   if ((p->flags & ~known) != 0u) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_LAMBDA_OVERRIDE) && !isfinite(p->lambda_override)) return ECOKV_ERR_INVALID_ARG;
   if (p->d != kD) return ECOKV_ERR_UNSUPPORTED;

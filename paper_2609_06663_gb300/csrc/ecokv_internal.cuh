@@ -70,6 +70,7 @@ struct ScoreArgs {
   const void* K;
   const void* Q;
   int N, W, g, R, h_kv, h_q, Tv, nchunks, p1_stride, ustat_stride;
+  int kbar_n;        // keys 0 .. kbar_n - 1 form the centroid (N, or Tv for the non-window centroid)
   float scale_log2;  // log2(e) / sqrt(d): logits are kept in log2 units
   float* p1part;
   float* ustat;

@@ -267,7 +267,7 @@ __global__ void __launch_bounds__(kThreads) pass1_kernel(ScoreArgs a) {
     float sk = 0.f, skh = 0.f;
     for (int r = 0; r < kChunk; ++r) {
       const float v = to_f32(ks[r * Tile<T>::stride + t]);
-      sk += v;
+      if (i0 + r < a.kbar_n) sk += v;  // the centroid's keys (all, or the candidates only)
       skh = fmaf(v, invn[r], skh);
     }
     part[2 * a.R + t] = sk;
@@ -290,7 +290,7 @@ __global__ void __launch_bounds__(kThreads) pass1_kernel(ScoreArgs a) {
     skh += __ldcg(base + (size_t)c * a.p1_stride + 2 * a.R + kD + t);
   }
   const float inv_n = 1.f / (float)a.N;
-  const float kb = sk * inv_n, mu = skh * inv_n;
+  const float kb = sk * (1.f / (float)a.kbar_n), mu = skh * inv_n;
   us[ustat_kbar() + t] = kb;
   us[ustat_mu() + t] = mu;
   for (int row = t; row < a.R; row += kThreads) {

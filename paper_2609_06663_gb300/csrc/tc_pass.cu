@@ -285,8 +285,8 @@ __device__ void unit_reduce_warp(const TcArgs& a, int u, int lane) {
         sh.x += hv[j].x; sh.y += hv[j].y; sh.z += hv[j].z; sh.w += hv[j].w;
       }
   }
-  const float inv_n = 1.f / (float)a.N;
-  const float4 kb = make_float4(sk.x * inv_n, sk.y * inv_n, sk.z * inv_n, sk.w * inv_n);
+  const float inv_n = 1.f / (float)a.N, inv_k = 1.f / (float)a.kbar_n;
+  const float4 kb = make_float4(sk.x * inv_k, sk.y * inv_k, sk.z * inv_k, sk.w * inv_k);
   const float4 mu = make_float4(sh.x * inv_n, sh.y * inv_n, sh.z * inv_n, sh.w * inv_n);
   reinterpret_cast<float4*>(us + ustat_kbar())[lane] = kb;
   reinterpret_cast<float4*>(us + ustat_mu())[lane] = mu;
@@ -976,6 +976,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const __nv_bfloat16 wlo = __float2bfloat16_rn(r1 - __bfloat162float(wmid));
           uint8_t* base = s.wbuf[stage] + (kk >> 6) * 2048 + (kk & 7) * 2;
           const int j = (kk & 63) >> 3;
+          if (a.kbar_n < a.N)  // non-window centroid: the window keys leave the sum of k
+            *reinterpret_cast<__nv_bfloat16*>(base + sw128(0, j)) = __float2bfloat16_rn(i < a.kbar_n ? 1.f : 0.f);
           *reinterpret_cast<__nv_bfloat16*>(base + sw128(1, j)) = whi;
           *reinterpret_cast<__nv_bfloat16*>(base + sw128(2, j)) = wmid;
           *reinterpret_cast<__nv_bfloat16*>(base + sw128(3, j)) = wlo;

@@ -12,6 +12,7 @@ constexpr int kTcP2Parts = 4;                  // parts a tail pass-2 item is sp
 
 struct TcArgs {
   int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
+  int kbar_n;                       // keys 0 .. kbar_n - 1 form the centroid (N, or Tv for the non-window centroid)
   int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int tiles_per_chunk, nchunks;     // chunks of kTcChunk keys per unit
   int lag_p2;                       // schedule lag (in units) of pass 2 behind pass 1 (<= U)

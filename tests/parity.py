@@ -15,7 +15,8 @@ TOL = {"f32": 1e-5, "bf16": 1e-3}
 def oracle_params(p, **over) -> O.Params:
     kw = {k: getattr(p, k) for k in ("n_layers", "h_kv", "h_q", "n", "d", "window", "budget", "pool_kernel",
                                       "alpha", "beta", "tau", "eps", "flags", "lambda_override")}
-    kw["flags"] = kw["flags"] & (O.FLAG_SC_MIXKV_SIGN | O.FLAG_LAMBDA_OVERRIDE | O.FLAG_VNORM_IMP)  # path flags mean nothing here
+    kw["flags"] = kw["flags"] & (O.FLAG_SC_MIXKV_SIGN | O.FLAG_LAMBDA_OVERRIDE | O.FLAG_VNORM_IMP |
+                                 O.FLAG_CENTROID_NONWIN)  # path flags mean nothing here
     kw.update(over)
     return O.Params(**kw)
 

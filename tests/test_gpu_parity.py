@@ -218,3 +218,18 @@ def test_c3_full_size_sampled_units():
         check_rows(K[l, h], idx[l, h], Ko[l, h], what)
         check_rows(V[l, h], idx[l, h], Vo[l, h], what)
     del op
+
+
+# the non-window centroid (reading R19): both streaming paths against the oracle
+@pytest.mark.parametrize("w,flags", [
+    (small_workload(5000, h_kv=2, group=4, window=8, budget=500, dtype="bf16", n_layers=2, clustered=True), 0),
+    (small_workload(5000, h_kv=2, group=4, window=8, budget=500, dtype="bf16", clustered=True),
+     E.ECOKV_FLAG_FORCE_SIMT),
+    (small_workload(3001, h_kv=2, group=1, window=8, budget=300, pool_kernel=7, dtype="f32"), 0),
+], ids=["bf16_tc", "bf16_simt", "f32_simt"])
+def test_non_window_centroid(w, flags):
+    run_and_compare(w, flags=flags | E.ECOKV_FLAG_CENTROID_NONWIN)
+
+
+def test_non_window_centroid_c2_two_layers():
+    run_and_compare(CONFIGS["c2"], layers=range(3, 5), flags=E.ECOKV_FLAG_CENTROID_NONWIN)

@@ -458,6 +458,25 @@ def test_pyramid_uniform_when_beta_is_one_and_integer_reading():
     assert O.pyramid_budgets(4, 10, 100.0, 8)[-1] == 8                # raised to the window
 
 
+def test_non_window_centroid_ignores_the_window_keys():
+    # with the non-window centroid, moving the window keys leaves the
+    # candidates' distances and s_E unchanged; with the default centroid they move
+    r = rng(26)
+    n, d, w = 50, 16, 6
+    K, u = aniso(r, n, d)
+    Qg = 4 * u + r.standard_normal((2, w, d))
+    K2 = K.copy()
+    K2[n - w:] += 7.0 * r.standard_normal((w, d))
+    nonwin = params(n, d, window=w, budget=20, h_q=2, pool=3, flags=O.FLAG_CENTROID_NONWIN)
+    a, b = O.score_head(K, Qg, nonwin), O.score_head(K2, Qg, nonwin)
+    assert np.allclose(a["d_e"], b["d_e"], rtol=1e-12, atol=0) and np.allclose(a["s_E"], b["s_E"], rtol=1e-12)
+    assert np.allclose(a["kbar"], K[:n - w].mean(axis=0), rtol=1e-12)
+    base = params(n, d, window=w, budget=20, h_q=2, pool=3)
+    c, e = O.score_head(K, Qg, base), O.score_head(K2, Qg, base)
+    assert not np.allclose(c["d_e"], e["d_e"], rtol=1e-6)
+    assert np.allclose(a["mu"], c["mu"]) and a["r_C"] == c["r_C"]        # the cosine terms keep all N
+
+
 def test_compact_rows():
     r = rng(18)
     X = r.standard_normal((12, 5))
