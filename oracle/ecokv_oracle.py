@@ -70,6 +70,12 @@ listed with its justification in the design notes):
       Algorithm 1 step 5): kbar over the T_v candidates (all N keys when
       T_v = 0); d_E of every key to that centroid, D_E still over all N (Eq.
       4); mu and r_C unchanged.
+  R20 Winsorised min-max of Eq. 2 (FLAG_WINSOR_1 / FLAG_WINSOR_5, the
+      normalisation ablation of Appendix B): q_lo and q_hi are order
+      statistics of d_E over the candidates, the floor(p (T_v - 1))-th and
+      the ceil((1 - p) (T_v - 1))-th smallest (0-based; p = 0.01 or 0.05, no
+      interpolation); s_E = (clip(d_E, q_lo, q_hi) - q_lo) / (q_hi - q_lo + eps).
+      The min-max of S_div in the rescale stays plain.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -87,6 +93,8 @@ FLAG_SC_MIXKV_SIGN = 0x1
 FLAG_LAMBDA_OVERRIDE = 0x2
 FLAG_VNORM_IMP = 0x4
 FLAG_CENTROID_NONWIN = 0x8
+FLAG_WINSOR_1 = 0x10   # 1 %-99 % winsorised min-max of Eq. 2
+FLAG_WINSOR_5 = 0x20   # 5 %-95 %
 
 NORM_FLOOR = 1e-12
 
@@ -188,6 +196,16 @@ def minmax(x: np.ndarray, eps: float) -> np.ndarray:
     """(x - min x) / (max x - min x + eps) (Eq. 2)."""
     lo, hi = x.min(), x.max()
     return (x - lo) / (hi - lo + eps)
+
+
+def winsor_minmax(x: np.ndarray, p: float, eps: float) -> np.ndarray:
+    """Winsorised min-max (R20): clip to the p and 1 - p order statistics,
+    then min-max between them."""
+    t = x.shape[0]
+    srt = np.sort(x)
+    lo = srt[int(np.floor(p * (t - 1)))]
+    hi = srt[int(np.ceil((1.0 - p) * (t - 1)))]
+    return (np.clip(x, lo, hi) - lo) / (hi - lo + eps)
 
 
 def euclid_redundancy(mean_dist: float, tau: float) -> float:
@@ -333,7 +351,10 @@ def score_head(K: np.ndarray, Qg: np.ndarray, p: Params, V: np.ndarray | None = 
 
     c = cosine_to_mean(KN[:t_v], mu)
     s_C = cosine_diversity(c, p.flags)
-    s_E = minmax(d_e_all[:t_v], p.eps)                             # Eq. 2
+    if p.flags & (FLAG_WINSOR_1 | FLAG_WINSOR_5):
+        s_E = winsor_minmax(d_e_all[:t_v], 0.01 if p.flags & FLAG_WINSOR_1 else 0.05, p.eps)   # R20
+    else:
+        s_E = minmax(d_e_all[:t_v], p.eps)                         # Eq. 2
     s_div = p.alpha * s_E + (1.0 - p.alpha) * s_C                 # Eq. 3
     s_tilde = rescale_diversity(s_div, s_imp, p.eps)
     S = lam * s_tilde + (1.0 - lam) * s_imp                        # Eq. 7

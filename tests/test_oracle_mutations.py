@@ -147,6 +147,11 @@ def pyramid_step_over_m(m, b_total, beta):      # slope divided by m, not m - 1
     return [b_first - (b_first - b_last) / m * l for l in range(m)]
 
 
+def winsor_interpolated(x, p, eps):        # percentiles interpolated instead of order statistics
+    lo, hi = np.percentile(x, 100 * p), np.percentile(x, 100 * (1 - p))
+    return (np.clip(x, lo, hi) - lo) / (hi - lo + eps)
+
+
 MUTANTS = {
     "no_scale": ("window_logits", no_scale),
     "no_causal_mask": ("window_logits", no_causal_mask),
@@ -168,6 +173,7 @@ MUTANTS = {
     "value_norm_squared": ("value_norms", value_norm_squared),
     "pyramid_top_without_m": ("pyramid_budgets_real", pyramid_top_without_m),
     "pyramid_step_over_m": ("pyramid_budgets_real", pyramid_step_over_m),
+    "winsor_interpolated": ("winsor_minmax", winsor_interpolated),
 }
 
 

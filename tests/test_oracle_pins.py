@@ -477,6 +477,22 @@ def test_non_window_centroid_ignores_the_window_keys():
     assert np.allclose(a["mu"], c["mu"]) and a["r_C"] == c["r_C"]        # the cosine terms keep all N
 
 
+def test_winsorised_minmax_closed_forms_and_outlier_invariance():
+    x = np.arange(100, dtype=float)                        # order statistics are the values
+    assert np.allclose(O.winsor_minmax(x, 0.01, 1e-6), O.minmax(x, 1e-6))   # 1 %: ranks 0 and 99
+    y = O.winsor_minmax(x, 0.05, 0.0)                      # 5 %: ranks floor(4.95) = 4, ceil(94.05) = 95
+    assert (y[:5] == 0).all() and (y[95:] == 1).all()
+    assert np.allclose(y[5:95], (x[5:95] - 4) / 91)
+    r = rng(27)
+    z = r.random(200)
+    w = z.copy()
+    w[17] = 1e9                                            # one extreme outlier
+    a, b = O.winsor_minmax(z, 0.05, 1e-6), O.winsor_minmax(w, 0.05, 1e-6)
+    keep = np.arange(200) != 17
+    assert np.allclose(a[keep], b[keep], rtol=0, atol=0.02) and b[17] == pytest.approx(1.0, abs=1e-5)
+    assert not np.allclose(O.minmax(z, 1e-6)[keep], O.minmax(w, 1e-6)[keep], atol=0.02)
+
+
 def test_compact_rows():
     r = rng(18)
     X = r.standard_normal((12, 5))
