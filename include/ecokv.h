@@ -74,6 +74,11 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
 #define ECOKV_FLAG_CENTROID_NONWIN 0x8u /* the centroid kbar of Eq. 1 over the n - window candidates only
                                             (Appendix B's alternative to Algorithm 1 step 5; all keys when
                                             n = window); d_E, D_E, mu and r_C otherwise as by default */
+#define ECOKV_FLAG_WINSOR_1        0x10u /* winsorised min-max of Eq. 2: d_E clipped to its order statistics
+                                             floor(p (n - W - 1)) and ceil((1 - p)(n - W - 1)) (0-based, no
+                                             interpolation), p = 1 % (Appendix B's normalisation ablation) */
+#define ECOKV_FLAG_WINSOR_5        0x20u /* the same with p = 5 %; at most one of the two.  Both: heads of up
+                                             to 32768 candidates, else ECOKV_ERR_UNSUPPORTED */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 
 typedef struct {

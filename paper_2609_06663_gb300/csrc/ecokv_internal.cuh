@@ -52,6 +52,7 @@ struct Layout {
   size_t chosen, src;  // layer-wide budget: chosen positions, gathered rows (U * min(B, N) int32 each)
   size_t lsel;         // layer-wide budget: the layer select's histograms, state and block counts
   size_t vnorm;        // value-norm importance: ||v_i|| of the candidates, U * Tv floats
+  size_t wins;         // winsorised min-max: the order statistics' selection state and histograms
   size_t total;
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
@@ -99,6 +100,10 @@ struct FinalArgs {
   float* dbg;        // [U][5][Tv] or null
   int32_t* idx;      // [U][n_keep] or null
   const float* vnorm;  // [U][Tv] ||v_i|| multiplying the pooled vote (value-norm importance), or null
+  // winsorised min-max: per unit the order-preserving keys of the clip
+  // bounds of d_E, at wlo[4 u] and whi[4 u]; null for the plain min-max
+  const unsigned* wlo;
+  const unsigned* whi;
   // per-layer budgets (PyramidKV schedule): with n_lb > 0 the heads of layer
   // l keep lb[l] rows (window included) in slots of stride n_keep
   int h_kv, n_lb;
@@ -147,6 +152,9 @@ cudaError_t launch_value_norms(const void* V, ecokv_dtype dt, int U, int N, int 
 bool cluster_finalize_fits(int Tv);
 // k largest of each layer's T scores, ascending positions (layer_select.cu)
 size_t layer_select_scratch_bytes(int n_layers, int T);
+// the k-th largest of each row's T values (its order-preserving key at
+// state[4 row]); hist: rows * 2048 unsigned, state: rows * 4 unsigned
+cudaError_t launch_row_kth(const float* S, int rows, int T, int k, unsigned* hist, unsigned* state, cudaStream_t s);
 cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int32_t* chosen, void* scratch,
                                 cudaStream_t s);
 // One thread-block cluster per unit: scores, and the top-k when f.idx is set

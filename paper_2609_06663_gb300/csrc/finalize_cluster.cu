@@ -68,12 +68,15 @@ struct ClusterSmem {
   unsigned hall[2][Shape<kJ>::kMaxCluster][256];
   float ext_all[Shape<kJ>::kMaxCluster][2];
   double simp_all[Shape<kJ>::kMaxCluster];  // value-norm importance: every rank's sum of S_imp
+  double wsum_all[Shape<kJ>::kMaxCluster];  // winsorised min-max: every rank's sum of the clipped d_E
   int cnt_all[Shape<kJ>::kMaxCluster][2];
   float red[kCWarps][8];  // per-warp partials
   float edge[32];         // pooling edge values
   float sc[8];            // broadcast scalars
   double dsc[2];          // sums behind the means of S_imp and of S_div
   double dred[kCWarps];   // per-warp sums of S_imp (value-norm importance)
+  double dredw[kCWarps];  // per-warp sums of the clipped d_E (winsorised min-max)
+  float wmax;             // winsorised min-max: the upper clip bound
   unsigned wsum[kCWarps];
   int wscan[kCWarps][2];  // per-warp counts above / equal to the threshold
   int shi[4];
@@ -88,6 +91,11 @@ __device__ __forceinline__ float sdiv_rcp(float dE, float c, float mnE, float in
   return __fadd_rn(__fmul_rn(alpha, sE), __fmul_rn(__fsub_rn(1.f, alpha), sC));
 }
 
+// The float an order-preserving key stands for (the inverse of ordered_key).
+__device__ __forceinline__ float key_float(unsigned k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 // Store v into the same object of every CTA of the cluster (its own included).
 template <int kMaxC, typename T>
 __device__ __forceinline__ void push_all(cg::cluster_group& cl, T* obj, T v, int C) {
@@ -97,7 +105,10 @@ __device__ __forceinline__ void push_all(cg::cluster_group& cl, T* obj, T v, int
 }
 
 // kMode: 0 = scores, 1 = scores and top-k, 2 = top-k of given scores (f.S).
-template <int kMode, int kJ>
+// kVar: the value-norm importance and winsorised min-max variants are compiled
+// in (their code is left out of the default kernel, whose register budget it
+// would cost).
+template <int kMode, int kJ, bool kVar>
 __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArgs f) {
   constexpr bool kSelect = kMode != 0;
   constexpr int kCap = Shape<kJ>::kCap, kMaxC = Shape<kJ>::kMaxCluster;
@@ -254,6 +265,11 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         s_c += sm.red[w][4];
         s_raw += sm.red[w][5];
       }
+      if (kVar && f.wlo != nullptr) {  // winsorised min-max: the order statistics replace the extrema
+        mnE = key_float(f.wlo[4 * u]);
+        mxE = key_float(f.whi[4 * u]);
+      }
+      sm.wmax = mxE;
       sm.sc[0] = s_all;
       sm.sc[1] = mnE;
       sm.sc[2] = __fadd_rn(__fsub_rn(mxE, mnE), f.eps);
@@ -265,7 +281,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     __syncthreads();
     const float mnE = sm.sc[1], denE = sm.sc[2];
     const float invE = __frcp_rn(denE);
-    if (f.vnorm != nullptr) {
+    if (kVar && f.vnorm != nullptr) {
       // value-norm importance: S_imp = pooled vote * ||v||, the norms staged
       // in coalesced order where the raw votes were; the sum of S_imp (its
       // mean is no longer a function of the raw-vote sums) goes round the
@@ -332,6 +348,9 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     //    and staged where the raw votes were, and its extrema over the
     //    cluster
     float mnD = INFINITY, mxD = -INFINITY;
+    const bool wins = kVar && f.wlo != nullptr;
+    const float wmax = sm.wmax;
+    double wsum = 0.0;  // winsorised min-max: this thread's sum of clipped d_E
     {
       const float* dEu = f.dE + (size_t)u * Tv;
       const float* cvu = f.cosv + (size_t)u * Tv;
@@ -355,6 +374,10 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   #pragma unroll
             for (int r = 0; r < 4; ++r)
               if (i + r < Tv) {
+                if (wins) {
+                  e[r] = fminf(fmaxf(e[r], mnE), wmax);
+                  wsum += (double)e[r];
+                }
                 const float sd = sdiv_rcp(e[r], cs[r], mnE, invE, f.alpha, mix);
                 sm.raw[pad_idx(i + r - lo + kHalo)] = sd;
                 mnD = fminf(mnD, sd);
@@ -367,13 +390,23 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         for (int j = 0; j < kJ; ++j) {
           const int i = lo + kCThreads * j + tid;
           if (i < Tv) {
-            const float sd = sdiv_rcp(__ldg(dEu + i), __ldg(cvu + i), mnE, invE, f.alpha, mix);
+            float e = __ldg(dEu + i);
+            if (wins) {
+              e = fminf(fmaxf(e, mnE), wmax);
+              wsum += (double)e;
+            }
+            const float sd = sdiv_rcp(e, __ldg(cvu + i), mnE, invE, f.alpha, mix);
             sm.raw[pad_idx(i - lo + kHalo)] = sd;
             mnD = fminf(mnD, sd);
             mxD = fmaxf(mxD, sd);
           }
         }
       }
+    }
+    if (wins) {
+  #pragma unroll
+      for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
+      if (lane == 0) sm.dredw[warp] = wsum;
     }
   #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -394,10 +427,15 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       }
       push_all<kMaxC>(cl, &sm.ext_all[rank][0], a0, C);
       push_all<kMaxC>(cl, &sm.ext_all[rank][1], a1, C);
-      if (f.vnorm != nullptr) {
+      if (kVar && f.vnorm != nullptr) {
         double cs = 0.0;
         for (int w = 0; w < kCWarps; ++w) cs += sm.dred[w];
         push_all<kMaxC>(cl, &sm.simp_all[rank], cs, C);
+      }
+      if (wins) {
+        double cs = 0.0;
+        for (int w = 0; w < kCWarps; ++w) cs += sm.dredw[w];
+        push_all<kMaxC>(cl, &sm.wsum_all[rank], cs, C);
       }
     }
     cl.sync();
@@ -409,11 +447,20 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       }
       const float denD = __fadd_rn(__fsub_rn(a1, a0), f.eps);
       // mean(S_imp) / mean(Sbar) with Sbar = (S_div - a0) / denD
-      const double num = sm.dsc[1] - (double)a0 * (double)Tv;  // Tv * denD * mean(Sbar)
+      double dsc1 = sm.dsc[1];  // Tv * mean(S_div)
+      if (wins) {  // s_E from the clipped distances: their sum replaces the sum of d_E
+        double sum_clip = 0.0;
+        for (int r = 0; r < C; ++r) sum_clip += sm.wsum_all[r];
+        const double T = (double)Tv, s_c = (double)sm.sc[4];
+        const double sum_sE = (sum_clip - (double)mnE * T) / (double)denE;
+        const double sum_sC = mix ? -s_c : (T - s_c) * 0.5;
+        dsc1 = (double)f.alpha * sum_sE + (1.0 - (double)f.alpha) * sum_sC;
+      }
+      const double num = dsc1 - (double)a0 * (double)Tv;  // Tv * denD * mean(Sbar)
       sm.sc[6] = a0;
       sm.sc[7] = denD;
       double dsc0 = sm.dsc[0];  // kp * Tv * mean(S_imp)
-      if (f.vnorm != nullptr) {
+      if (kVar && f.vnorm != nullptr) {
         double sum_imp = 0.0;
         for (int r = 0; r < C; ++r) sum_imp += sm.simp_all[r];
         dsc0 = (double)f.pool * sum_imp;
@@ -454,7 +501,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         dbg[Tv + i] = __fmul_rn(acc, inv_pool);
         dbg[2 * Tv + i] = e;
         dbg[3 * Tv + i] = cs;
-        dbg[4 * Tv + i] = sdiv_rcp(e, cs, mnE, invE, f.alpha, mix);
+        dbg[4 * Tv + i] = sdiv_rcp(wins ? fminf(fmaxf(e, mnE), wmax) : e, cs, mnE, invE, f.alpha, mix);
       }
     }
     if (f.S != nullptr) {
@@ -638,13 +685,17 @@ template <int kJ>
 cudaError_t set_smem_attrs() {
   const int bytes = (int)sizeof(ClusterSmem<kJ>);
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                bytes)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                bytes)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                bytes)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 bytes)) != cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                bytes)) != cudaSuccess)
-    return e;
-  return cudaFuncSetAttribute(finalize_cluster_kernel<2, kJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  return cudaFuncSetAttribute(finalize_cluster_kernel<2, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              bytes);
 }
 
 template <int kJ>
@@ -663,9 +714,13 @@ cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cud
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ>, f);
-  if (f.idx == nullptr) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ>, f);
-  return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ>, f);
+  const bool var = f.vnorm != nullptr || f.wlo != nullptr;
+  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ, false>, f);
+  if (f.idx == nullptr)
+    return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ, true>, f)
+               : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ, false>, f);
+  return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ, true>, f)
+             : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ, false>, f);
 }
 
 }  // namespace

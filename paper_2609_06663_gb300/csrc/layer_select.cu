@@ -259,4 +259,26 @@ cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int3
   return cudaSuccess;
 }
 
+cudaError_t launch_row_kth(const float* S, int rows, int T, int k, unsigned* hist, unsigned* state, cudaStream_t s) {
+  if (rows <= 0 || T <= 0 || k < 1 || k > T) return cudaErrorInvalidValue;
+  LsArgs a{};
+  a.S = S;
+  a.T = T;
+  a.k = k;
+  a.nblk = (T + kLsSpan - 1) / kLsSpan;
+  a.ghist = hist;
+  a.state = state;
+  cudaError_t e = cudaMemsetAsync(hist, 0, (size_t)rows * kLsMaxBins * 4, s);
+  if (e != cudaSuccess || (e = cudaMemsetAsync(state, 0, (size_t)rows * 4 * 4, s)) != cudaSuccess) return e;
+  const dim3 grid(a.nblk, rows), blk(kLsThreads);
+  if ((e = launch_dependent(ls_hist<11>, grid, blk, s, a, 21)) != cudaSuccess ||
+      (e = launch_dependent(ls_digit<11>, dim3(rows), dim3(256), s, a, 21, 1)) != cudaSuccess ||
+      (e = launch_dependent(ls_hist<11>, grid, blk, s, a, 10)) != cudaSuccess ||
+      (e = launch_dependent(ls_digit<11>, dim3(rows), dim3(256), s, a, 10, 0)) != cudaSuccess ||
+      (e = launch_dependent(ls_hist<10>, grid, blk, s, a, 0)) != cudaSuccess ||
+      (e = launch_dependent(ls_digit<10>, dim3(rows), dim3(256), s, a, 0, 0)) != cudaSuccess)
+    return e;
+  return cudaSuccess;
+}
+
 }  // namespace ecokv

@@ -233,3 +233,22 @@ def test_non_window_centroid(w, flags):
 
 def test_non_window_centroid_c2_two_layers():
     run_and_compare(CONFIGS["c2"], layers=range(3, 5), flags=E.ECOKV_FLAG_CENTROID_NONWIN)
+
+
+# winsorised min-max of Eq. 2 (reading R20): both streaming paths and both
+# clip levels against the oracle (scores, lambda, the per-token terms,
+# selection, rows)
+@pytest.mark.parametrize("w,flags", [
+    (small_workload(5000, h_kv=2, group=4, window=8, budget=500, dtype="bf16", n_layers=2, clustered=True),
+     E.ECOKV_FLAG_WINSOR_5),
+    (small_workload(20000, h_kv=2, group=4, window=8, budget=2000, dtype="bf16", clustered=True),
+     E.ECOKV_FLAG_WINSOR_1),
+    (small_workload(3001, h_kv=2, group=1, window=8, budget=300, pool_kernel=7, dtype="f32"),
+     E.ECOKV_FLAG_WINSOR_1),
+], ids=["bf16_tc_5pct", "bf16_wide_1pct", "f32_simt_1pct"])
+def test_winsorised_minmax(w, flags):
+    run_and_compare(w, flags=flags)
+
+
+def test_winsorised_minmax_c2_two_layers():
+    run_and_compare(CONFIGS["c2"], layers=range(10, 12), flags=E.ECOKV_FLAG_WINSOR_5)
