@@ -1,9 +1,9 @@
 """CUDA path (through the C ABI) vs the fp64 oracle on the same seeded inputs.
 
 Small shapes span several 128-key chunks and a ragged tail; the configs run
-at their own shapes (layer subsets where the oracle would take long), and the
-32k-token config runs at full size in the same launch the benchmark times,
-checked on sampled (layer, head) units."""
+at their own shapes (layer subsets where the oracle would take long), and
+every bf16 config also runs at full size in one call (the 32k-token one in
+the same launch the benchmark times), checked on sampled (layer, head) units."""
 import numpy as np
 import pytest
 import torch
@@ -196,28 +196,33 @@ def test_compact_reports_bad_index():
     assert torch.equal(Ko[0, 0], Kd[0, 0][good])
 
 
-def test_c3_full_size_sampled_units():
-    # the 32k-token, 28-layer workload exactly as the benchmark launches it
-    w = workload("c3_b10")
+@pytest.mark.parametrize("key,units", [
+    ("c3_b10", [(0, 0), (13, 2), (27, 3)]),      # as the benchmark launches it
+    ("c3_b5", [(5, 1), (27, 0)]),
+    ("c3_b20", [(0, 3), (20, 2)]),
+    ("c2", [(0, 0), (17, 3), (27, 1)]),
+    ("c1_b10", [(0, 0), (16, 31), (31, 7)]),
+])
+def test_full_size_sampled_units(key, units):
+    # every layer and head of the configuration in one call, at full size;
+    # sampled heads against the oracle
+    w = workload(key)
     K, V, Q = make_inputs(w, device=DEV)
     p = params_of(w)
     ws = E.alloc_workspace(p, DEV)
     idx, Ko, Vo, S, lam = E.evict(p, K, V, Q, ws=ws, want_scores=True)
     torch.cuda.synchronize()
     assert E.ecokv_device_status(ws) == 0
-    units = [(0, 0), (13, 2), (27, 3)]
-    op = oracle_params(p, n_layers=1)
+    tol = TOL[w.dtype]
     for (l, h) in units:
         Kh = K[l:l + 1, h:h + 1].cpu()
         Qh = Q[l:l + 1, h * w.group:(h + 1) * w.group].cpu()
         r = O.evict(Kh, Kh, Qh, oracle_params(p, n_layers=1, h_kv=1, h_q=w.group))[(0, 0)]
-        what = f"c3 unit ({l},{h})"
-        check_scores(S[l, h].cpu().double().numpy(), r, TOL["bf16"], what)
-        check_selection(idx[l, h].cpu().numpy(), r, oracle_params(p, n_layers=1, h_kv=1, h_q=w.group),
-                        TOL["bf16"], what)
+        what = f"{key} unit ({l},{h})"
+        check_scores(S[l, h].cpu().double().numpy(), r, tol, what)
+        check_selection(idx[l, h].cpu().numpy(), r, oracle_params(p, n_layers=1, h_kv=1, h_q=w.group), tol, what)
         check_rows(K[l, h], idx[l, h], Ko[l, h], what)
         check_rows(V[l, h], idx[l, h], Vo[l, h], what)
-    del op
 
 
 # the non-window centroid (reading R19): both streaming paths against the oracle
