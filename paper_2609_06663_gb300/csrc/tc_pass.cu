@@ -772,8 +772,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (ok) {
             mbar_expect_tx(&s.full[stage], kTileBytes);
             const int y = i0 + t * kTile;
-            // pass 1 keeps its keys in L2 for pass 2; pass 2 reads them for the last time
-            const uint64_t pol = it.type == kP1 ? pol_keep : pol_drop;
+            // with pass 2 close behind pass 1 (a short lag), pass 1 keeps its
+            // keys in L2 for it; with all of pass 1 first no key survives in L2
+            // until its pass 2, and keeping them only crowds out the data the
+            // finalisation reads next, so every load is evict-first
+            const uint64_t pol = (it.type == kP1 && a.lag_p2 < a.U) ? pol_keep : pol_drop;
             tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u, pol);
             tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u, pol);
             used_bits |= 1u << stage;
