@@ -351,8 +351,8 @@ __device__ void gather_rows(const CompactArgs& a, int u, int r0, int r1, int tid
         const int src = __ldcg(idx + r);
         dst[j] = r * vpr + v;
         if (src >= 0 && src < a.N) {
-          kv[j] = __ldg(K + (size_t)src * vpr + v);
-          vv[j] = __ldg(V + (size_t)src * vpr + v);
+          kv[j] = __ldcs(K + (size_t)src * vpr + v);  // each row is read once
+          vv[j] = __ldcs(V + (size_t)src * vpr + v);
         } else if (a.status != nullptr) {
           atomicCAS(a.status, 0u, (unsigned)ECOKV_ERR_DEVICE_INDEX);
           a.status[1] = (unsigned)u;
@@ -362,8 +362,8 @@ __device__ void gather_rows(const CompactArgs& a, int u, int r0, int r1, int tid
 #pragma unroll
     for (int j = 0; j < 4; ++j)
       if (dst[j] >= 0) {
-        Ko[dst[j]] = kv[j];
-        Vo[dst[j]] = vv[j];
+        __stcs(Ko + dst[j], kv[j]);
+        __stcs(Vo + dst[j], vv[j]);
       }
   }
 }

@@ -971,7 +971,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float n2 = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
-          if (valid) a.norm2[(size_t)u * a.N + i] = n2;
+          if (valid) __stcs(a.norm2 + (size_t)u * a.N + i, n2);  // read once, by pass 2
           const float w = valid ? rsqrtf(fmaxf(n2, 1e-24f)) : 0.f;
           const __nv_bfloat16 whi = __float2bfloat16_rn(w);
           const float r1 = w - __bfloat162float(whi);
@@ -994,7 +994,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(&s.empty[stage]);
           const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
           ++p2count;
-          const float n2 = valid ? __ldcg(a.norm2 + (size_t)u * a.N + i) : 0.f;
+          const float n2 = valid ? __ldcs(a.norm2 + (size_t)u * a.N + i) : 0.f;
           if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u)))) break;
           s.nbuf[nb][kk] = n2;
           __syncwarp();
