@@ -49,7 +49,7 @@ Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
   L.src = off;     off += align256(U * n_keep * 4);
   L.lsel = off;    off += align256(layer_select_scratch_bytes(p.n_layers, p.h_kv * L.Tv));
   L.vnorm = off;   off += align256(U * (size_t)L.Tv * 4);
-  L.wins = off;    off += align256(U * (2048 + 8) * 4);
+  L.wins = off;    off += align256(U * 2 * (2048 + 4) * 4);
   L.total = off;
   return L;
 }
@@ -287,12 +287,10 @@ static ecokv_status winsor_launch(const ecokv_params& p, const Layout& L, char* 
   const double q = (p.flags & ECOKV_FLAG_WINSOR_1) ? 0.01 : 0.05;
   const int r_lo = (int)floor(q * (double)(L.Tv - 1)), r_hi = (int)ceil((1.0 - q) * (double)(L.Tv - 1));
   unsigned* hist = reinterpret_cast<unsigned*>(ws + L.wins);
-  unsigned* lo = hist + (size_t)L.U * 2048;
+  unsigned* lo = hist + (size_t)2 * L.U * 2048;
   unsigned* hi = lo + (size_t)L.U * 4;
   const float* dE = reinterpret_cast<const float*>(ws + L.dE);
-  if (launch_row_kth(dE, L.U, L.Tv, L.Tv - r_lo, hist, lo, s) != cudaSuccess ||
-      launch_row_kth(dE, L.U, L.Tv, L.Tv - r_hi, hist, hi, s) != cudaSuccess)
-    return ECOKV_ERR_CUDA;
+  if (launch_row_kth2(dE, L.U, L.Tv, L.Tv - r_lo, L.Tv - r_hi, hist, lo, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   f.wlo = lo;
   f.whi = hi;
   return ECOKV_OK;

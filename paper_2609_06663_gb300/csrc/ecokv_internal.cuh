@@ -152,9 +152,11 @@ cudaError_t launch_value_norms(const void* V, ecokv_dtype dt, int U, int N, int 
 bool cluster_finalize_fits(int Tv);
 // k largest of each layer's T scores, ascending positions (layer_select.cu)
 size_t layer_select_scratch_bytes(int n_layers, int T);
-// the k-th largest of each row's T values (its order-preserving key at
-// state[4 row]); hist: rows * 2048 unsigned, state: rows * 4 unsigned
-cudaError_t launch_row_kth(const float* S, int rows, int T, int k, unsigned* hist, unsigned* state, cudaStream_t s);
+// the k1-th and the k2-th largest of each row's T values (their
+// order-preserving keys at state[4 row] and state[4 (rows + row)]);
+// hist: 2 * rows * 2048 unsigned, state: 2 * rows * 4 unsigned
+cudaError_t launch_row_kth2(const float* S, int rows, int T, int k1, int k2, unsigned* hist, unsigned* state,
+                            cudaStream_t s);
 cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int32_t* chosen, void* scratch,
                                 cudaStream_t s);
 // One thread-block cluster per unit: scores, and the top-k when f.idx is set
