@@ -120,6 +120,19 @@ def test_pyramid_budgets_and_layered_entry_reject_bad_arguments(lib):
                                  ws) == 1
 
 
+def test_adaptive_entry_rejects_bad_arguments(lib):
+    p = good()
+    fake = 1 << 20
+    ws = E.ecokv_workspace_size(p)
+    # head offsets missing, then misaligned
+    assert E.ecokv_evict_adaptive(p, 1, fake, fake, fake, fake, None, fake, fake, None, fake, ws) == 1
+    assert E.ecokv_evict_adaptive(p, 1, fake, fake, fake, fake, fake + 2, fake, fake, None, fake, ws) == 1
+    assert E.ecokv_evict_adaptive(p, 1, fake, fake, fake, fake, fake, fake, fake, None, fake, ws - 1) == 3
+    # both winsorising levels at once
+    p.flags = E.ECOKV_FLAG_WINSOR_1 | E.ECOKV_FLAG_WINSOR_5
+    assert E.ecokv_check_params(p) == 1
+
+
 def test_status_strings(lib):
     for c in range(7):
         assert E.ecokv_status_string(c)
