@@ -76,6 +76,14 @@ listed with its justification in the design notes):
       the ceil((1 - p) (T_v - 1))-th smallest (0-based; p = 0.01 or 0.05, no
       interpolation); s_E = (clip(d_E, q_lo, q_hi) - q_lo) / (q_hi - q_lo + eps).
       The min-max of S_div in the rescale stays plain.
+  R21 MAD scaling of Eq. 2 (FLAG_MAD; the same ablation names per-head MAD
+      scaling at temperature 1 without its formula): med = median of d_E over
+      the candidates, MAD = median of |d_E - med| (a median of an even count
+      is the mean of its two middle order statistics); s_E = sigma((d_E -
+      med) / (MAD + eps)), the logistic function at temperature 1 mapping the
+      robust z-score into (0, 1), the range Eq. 2's text gives the diversity
+      scores.  The min-max of S_div stays plain; at most one of FLAG_MAD and
+      the winsorising flags.
 
 Parity pins: every function below is checked in tests/test_oracle_pins.py
 against closed forms, invariants, special cases that reduce to a library
@@ -95,6 +103,7 @@ FLAG_VNORM_IMP = 0x4
 FLAG_CENTROID_NONWIN = 0x8
 FLAG_WINSOR_1 = 0x10   # 1 %-99 % winsorised min-max of Eq. 2
 FLAG_WINSOR_5 = 0x20   # 5 %-95 %
+FLAG_MAD = 0x40        # MAD scaling of Eq. 2
 
 NORM_FLOOR = 1e-12
 
@@ -206,6 +215,16 @@ def winsor_minmax(x: np.ndarray, p: float, eps: float) -> np.ndarray:
     lo = srt[int(np.floor(p * (t - 1)))]
     hi = srt[int(np.ceil((1.0 - p) * (t - 1)))]
     return (np.clip(x, lo, hi) - lo) / (hi - lo + eps)
+
+
+def mad_scale(x: np.ndarray, eps: float) -> np.ndarray:
+    """Per-head MAD scaling (R21): the logistic function of (x - median x) /
+    (MAD + eps), MAD the median absolute deviation from the median."""
+    med = np.median(x)
+    mad = np.median(np.abs(x - med))
+    z = (x - med) / (mad + eps)
+    with np.errstate(over="ignore"):
+        return 1.0 / (1.0 + np.exp(-z))
 
 
 def euclid_redundancy(mean_dist: float, tau: float) -> float:
@@ -353,6 +372,8 @@ def score_head(K: np.ndarray, Qg: np.ndarray, p: Params, V: np.ndarray | None = 
     s_C = cosine_diversity(c, p.flags)
     if p.flags & (FLAG_WINSOR_1 | FLAG_WINSOR_5):
         s_E = winsor_minmax(d_e_all[:t_v], 0.01 if p.flags & FLAG_WINSOR_1 else 0.05, p.eps)   # R20
+    elif p.flags & FLAG_MAD:
+        s_E = mad_scale(d_e_all[:t_v], p.eps)                      # R21
     else:
         s_E = minmax(d_e_all[:t_v], p.eps)                         # Eq. 2
     s_div = p.alpha * s_E + (1.0 - p.alpha) * s_C                 # Eq. 3

@@ -152,6 +152,28 @@ def winsor_interpolated(x, p, eps):        # percentiles interpolated instead of
     return (np.clip(x, lo, hi) - lo) / (hi - lo + eps)
 
 
+def mad_lower_median(x, eps):              # the lower middle value as the median of an even count
+    srt = np.sort(x)
+    med = srt[(len(x) - 1) // 2]
+    dev = np.sort(np.abs(x - med))
+    mad = dev[(len(x) - 1) // 2]
+    return 1.0 / (1.0 + np.exp(-(x - med) / (mad + eps)))
+
+
+def mad_std_scale(x, eps):                 # mean and standard deviation instead of median and MAD
+    return 1.0 / (1.0 + np.exp(-(x - x.mean()) / (x.std() + eps)))
+
+
+def mad_signed_deviation(x, eps):          # median of x - med instead of |x - med|
+    med = np.median(x)
+    mad = np.median(x - med)
+    return 1.0 / (1.0 + np.exp(-(x - med) / (mad + eps)))
+
+
+def mad_flipped(x, eps):                   # logistic of -z
+    return 1.0 - ORIG["mad_scale"](x, eps)
+
+
 MUTANTS = {
     "no_scale": ("window_logits", no_scale),
     "no_causal_mask": ("window_logits", no_causal_mask),
@@ -174,6 +196,10 @@ MUTANTS = {
     "pyramid_top_without_m": ("pyramid_budgets_real", pyramid_top_without_m),
     "pyramid_step_over_m": ("pyramid_budgets_real", pyramid_step_over_m),
     "winsor_interpolated": ("winsor_minmax", winsor_interpolated),
+    "mad_lower_median": ("mad_scale", mad_lower_median),
+    "mad_std_scale": ("mad_scale", mad_std_scale),
+    "mad_signed_deviation": ("mad_scale", mad_signed_deviation),
+    "mad_flipped": ("mad_scale", mad_flipped),
 }
 
 

@@ -493,6 +493,62 @@ def test_winsorised_minmax_closed_forms_and_outlier_invariance():
     assert not np.allclose(O.minmax(z, 1e-6)[keep], O.minmax(w, 1e-6)[keep], atol=0.02)
 
 
+def test_mad_scaling_closed_forms():
+    # 0..100: median 50; the absolute deviations are 0 once and 1..50 twice,
+    # so their median (the 51st smallest) is 25
+    x = np.arange(101, dtype=float)
+    s = O.mad_scale(x, 0.0)
+    assert s[50] == 0.5
+    assert s[75] == pytest.approx(0.7310585786300049, rel=1e-14)     # logistic(1)
+    assert s[0] == pytest.approx(0.11920292202211755, rel=1e-14)     # logistic(-2)
+    assert s[100] == pytest.approx(0.8807970779778823, rel=1e-14)    # logistic(2)
+    # 0..99: median 49.5 (mean of the middle two); deviations 0.5 .. 49.5 twice
+    # each, median (24.5 + 25.5) / 2 = 25
+    y = np.arange(100, dtype=float)
+    t = O.mad_scale(y, 0.0)
+    assert t[62] == pytest.approx(0.6224593312018546, rel=1e-14)     # logistic(0.5)
+    assert t[37] == pytest.approx(0.3775406687981454, rel=1e-14)     # logistic(-0.5)
+    # eps enters the denominator
+    assert O.mad_scale(x, 25.0)[100] == pytest.approx(0.7310585786300049, rel=1e-14)
+
+
+def test_mad_scaling_invariances_and_outlier():
+    r = rng(28)
+    z = r.lognormal(0.0, 0.7, 301)
+    s = O.mad_scale(z, 0.0)
+    assert ((s > 0) & (s < 1)).all()
+    assert (np.argsort(s, kind="stable") == np.argsort(z, kind="stable")).all()     # order kept
+    assert np.allclose(O.mad_scale(3.5 * z + 11.0, 0.0), s, rtol=1e-12)          # affine invariant
+    assert np.sum(s > 0.5) == np.sum(s < 0.5) == 150                              # median maps to 1/2
+    assert O.mad_scale(np.full(9, 2.5), 1e-6).tolist() == [0.5] * 9               # MAD = 0
+    w = z.copy()
+    w[17] = 1e9
+    b = O.mad_scale(w, 0.0)
+    keep = np.arange(301) != 17
+    assert np.allclose(b[keep], s[keep], atol=0.02) and b[17] == 1.0
+    def std_scaled(v):                                     # a mean / std z-score is not robust to it
+        return 1.0 / (1.0 + np.exp(-(v - v.mean()) / v.std()))
+    assert not np.allclose(std_scaled(w)[keep], std_scaled(z)[keep], atol=0.02)
+
+
+def test_mad_flag_replaces_the_minmax_of_eq2():
+    # alpha = 1 and lambda = 1: S ranks the candidates by s_E; with the MAD
+    # flag the candidate at the median distance has s_E = 1/2 exactly
+    r = rng(29)
+    n, d, w = 41, 16, 4                                    # 37 candidates
+    K, u = aniso(r, n, d)
+    Qg = 4 * u + r.standard_normal((1, w, d))
+    pm = params(n, d, window=w, budget=12, pool=3, alpha=1.0, lambda_override=1.0,
+                flags=O.FLAG_MAD | O.FLAG_LAMBDA_OVERRIDE)
+    out = O.score_head(K, Qg, pm)
+    mid = np.argsort(out["d_e"])[18]
+    assert out["s_E"][mid] == 0.5
+    assert (np.argsort(out["S"]) == np.argsort(out["d_e"])).all()
+    plain = O.score_head(K, Qg, params(n, d, window=w, budget=12, pool=3, alpha=1.0, lambda_override=1.0,
+                                       flags=O.FLAG_LAMBDA_OVERRIDE))
+    assert plain["s_E"].min() == 0.0 and out["s_E"].min() > 0.0
+
+
 def test_compact_rows():
     r = rng(18)
     X = r.standard_normal((12, 5))
