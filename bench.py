@@ -49,12 +49,14 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=0,
                     help="run only this many layers of the workload (small profiling captures)")
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm", "pyramid", "centroid-nonwin", "winsor5"], default="per-head",
+    ap.add_argument("--variant", choices=["per-head", "adaptive", "vnorm", "pyramid", "centroid-nonwin", "winsor5", "mad"],
+                    default="per-head",
                     help="adaptive: layer-wide budget shared by a layer's heads (ecokv_evict_adaptive); "
                          "vnorm: importance weighted by the value norms (ECOKV_FLAG_VNORM_IMP); "
                          "pyramid: PyramidKV per-layer budgets, beta 20 (ecokv_evict_layered); "
                          "centroid-nonwin: the centroid over the candidates only (ECOKV_FLAG_CENTROID_NONWIN); "
-                         "winsor5: 5 %-95 % winsorised min-max of Eq. 2 (ECOKV_FLAG_WINSOR_5)")
+                         "winsor5: 5 %-95 % winsorised min-max of Eq. 2 (ECOKV_FLAG_WINSOR_5); "
+                         "mad: MAD scaling in place of the min-max of Eq. 2 (ECOKV_FLAG_MAD)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -308,7 +310,8 @@ def main():
                       budget=max(budgets) if budgets else w.budget, pool_kernel=w.pool_kernel,
                       flags={"vnorm": E.ECOKV_FLAG_VNORM_IMP,
                              "centroid-nonwin": E.ECOKV_FLAG_CENTROID_NONWIN,
-                             "winsor5": E.ECOKV_FLAG_WINSOR_5}.get(args.variant, 0))
+                             "winsor5": E.ECOKV_FLAG_WINSOR_5,
+                             "mad": E.ECOKV_FLAG_MAD}.get(args.variant, 0))
     ws = E.alloc_workspace(p, dev)
     n_keep = min(p.budget, w.n)
     idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
@@ -471,14 +474,16 @@ def main():
                                "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)",
                                "pyramid": f"per-layer budgets, PyramidKV beta 20: {budgets}",
                                "centroid-nonwin": "non-window centroid (ECOKV_FLAG_CENTROID_NONWIN)",
-                               "winsor5": "5 %-95 % winsorised min-max (ECOKV_FLAG_WINSOR_5)"}.get(
+                               "winsor5": "5 %-95 % winsorised min-max (ECOKV_FLAG_WINSOR_5)",
+                               "mad": "MAD scaling of d_E (ECOKV_FLAG_MAD)"}.get(
                                    args.variant, "per-head budget"),
                    "evicted_rows_per_s": round(job_rate(world, w.units * max(0, w.n - w.budget), ms_step), 1),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
         # the layer-wide budget adds the layer select (3 digits x 2, count, emit) and the split
         "gpu_launches": (launches_per_call(w) + (9 if adaptive else 0) + (1 if args.variant == "vnorm" else 0)
-                         + (12 if args.variant == "winsor5" else 0))
+                         # the robust forms of Eq. 2: one order-statistics launch
+                         + (1 if args.variant in ("winsor5", "mad") else 0))
         * args.steps, "clocks": clocks,
         "timing": {"headline": f"{args.steps} steps back to back, CUDA events around the region",
                    "stages": f"{args.steps} further steps with per-launch events (launches serialised)",

@@ -79,6 +79,12 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
                                              interpolation), p = 1 % (Appendix B's normalisation ablation) */
 #define ECOKV_FLAG_WINSOR_5        0x20u /* the same with p = 5 %; at most one of the two.  Both: heads of up
                                              to 32768 candidates, else ECOKV_ERR_UNSUPPORTED */
+#define ECOKV_FLAG_MAD             0x40u /* MAD scaling in place of the min-max of Eq. 2 (the same ablation):
+                                             s_E = logistic((d_E - med) / (MAD + eps)), med the median of d_E
+                                             over the candidates and MAD the median of |d_E - med| (an even
+                                             count's median is the mean of its two middle values).  Not with
+                                             a WINSOR flag (ECOKV_ERR_INVALID_ARG); heads of up to 32768
+                                             candidates, else ECOKV_ERR_UNSUPPORTED */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 
 typedef struct {

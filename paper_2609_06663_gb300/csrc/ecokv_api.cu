@@ -49,7 +49,7 @@ Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
   L.src = off;     off += align256(U * n_keep * 4);
   L.lsel = off;    off += align256(layer_select_scratch_bytes(p.n_layers, p.h_kv * L.Tv));
   L.vnorm = off;   off += align256(U * (size_t)L.Tv * 4);
-  L.wins = off;    off += align256(U * 2 * (2048 + 4) * 4);
+  L.wins = off;    off += align256(U * 4 * 4 * 4);
   L.total = off;
   return L;
 }
@@ -166,6 +166,7 @@ static FinalArgs final_args(const ecokv_params& p, const Layout& L, char* ws) {
   f.flags = p.flags;
   f.n_keep = p.budget < p.n ? p.budget : p.n;
   f.h_kv = p.h_kv;
+  f.n_units = L.U;
   if (ws != nullptr) {
     f.p2part = reinterpret_cast<const float*>(ws + L.p2part);
     f.ustat = reinterpret_cast<const float*>(ws + L.ustat);
@@ -274,25 +275,35 @@ static ecokv_status vnorm_launch(const ecokv_params& p, ecokv_dtype dt, const La
   return launch_value_norms(V, dt, L.U, p.n, L.Tv, vn, s) == cudaSuccess ? ECOKV_OK : ECOKV_ERR_CUDA;
 }
 
-// Winsorised min-max: the clip bounds of d_E per unit, the order statistics
-// floor(p (Tv - 1)) and ceil((1 - p)(Tv - 1)) (0-based ascending), found as
-// the (Tv - rank)-th largest by radix select over the pass-2 distances.
+// Order statistics of d_E for the robust forms of Eq. 2, found as
+// (Tv - rank)-th largest values by one radix-select launch (a CTA per unit)
+// over the pass-2 distances:
+// - winsorised min-max: the clip bounds, ranks floor(p (Tv - 1)) and
+//   ceil((1 - p)(Tv - 1)) (0-based ascending);
+// - MAD scaling: the two middle ranks floor((Tv - 1) / 2) and floor(Tv / 2)
+//   of d_E (their mean is the median), then the same ranks of |d_E - median|.
 static bool winsor(const ecokv_params& p) { return (p.flags & (ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5)) != 0; }
-static ecokv_status winsor_check(const ecokv_params& p, const Layout& L) {
-  if (!winsor(p)) return ECOKV_OK;
+static bool robust(const ecokv_params& p) { return winsor(p) || (p.flags & ECOKV_FLAG_MAD) != 0; }
+static ecokv_status robust_check(const ecokv_params& p, const Layout& L) {
+  if (!robust(p)) return ECOKV_OK;
   return cluster_finalize_fits(L.Tv) && L.Tv > 0 ? ECOKV_OK : ECOKV_ERR_UNSUPPORTED;
 }
-static ecokv_status winsor_launch(const ecokv_params& p, const Layout& L, char* ws, FinalArgs& f, cudaStream_t s) {
-  if (!winsor(p)) return ECOKV_OK;
-  const double q = (p.flags & ECOKV_FLAG_WINSOR_1) ? 0.01 : 0.05;
-  const int r_lo = (int)floor(q * (double)(L.Tv - 1)), r_hi = (int)ceil((1.0 - q) * (double)(L.Tv - 1));
-  unsigned* hist = reinterpret_cast<unsigned*>(ws + L.wins);
-  unsigned* lo = hist + (size_t)2 * L.U * 2048;
-  unsigned* hi = lo + (size_t)L.U * 4;
+static ecokv_status robust_launch(const ecokv_params& p, const Layout& L, char* ws, FinalArgs& f, cudaStream_t s) {
+  if (!robust(p)) return ECOKV_OK;
+  unsigned* st = reinterpret_cast<unsigned*>(ws + L.wins);  // [4][U][4]
   const float* dE = reinterpret_cast<const float*>(ws + L.dE);
-  if (launch_row_kth2(dE, L.U, L.Tv, L.Tv - r_lo, L.Tv - r_hi, hist, lo, s) != cudaSuccess) return ECOKV_ERR_CUDA;
-  f.wlo = lo;
-  f.whi = hi;
+  const int T = L.Tv;
+  if (winsor(p)) {
+    const double q = (p.flags & ECOKV_FLAG_WINSOR_1) ? 0.01 : 0.05;
+    const int r_lo = (int)floor(q * (double)(T - 1)), r_hi = (int)ceil((1.0 - q) * (double)(T - 1));
+    if (launch_order_stats(dE, L.U, T, T - r_lo, T - r_hi, false, st, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+    f.wlo = st;
+    f.whi = st + (size_t)L.U * 4;
+    return ECOKV_OK;
+  }
+  const int m_lo = (T - 1) / 2, m_hi = T / 2;
+  if (launch_order_stats(dE, L.U, T, T - m_lo, T - m_hi, true, st, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  f.mad = st;
   return ECOKV_OK;
 }
 
@@ -333,9 +344,11 @@ ecokv_status ecokv_check_params(const ecokv_params* p) {
   if (!(p->eps > 0.f) || !isfinite(p->eps) || !isfinite(p->tau)) return ECOKV_ERR_INVALID_ARG;
   const uint32_t known =
       ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_VNORM_IMP | ECOKV_FLAG_CENTROID_NONWIN |
-      ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5 | ECOKV_FLAG_FORCE_SIMT;
+      ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5 | ECOKV_FLAG_MAD | ECOKV_FLAG_FORCE_SIMT;
   if ((p->flags & ~known) != 0u) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_WINSOR_1) && (p->flags & ECOKV_FLAG_WINSOR_5)) return ECOKV_ERR_INVALID_ARG;
+  if ((p->flags & ECOKV_FLAG_MAD) && (p->flags & (ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5)))
+    return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_LAMBDA_OVERRIDE) && !isfinite(p->lambda_override)) return ECOKV_ERR_INVALID_ARG;
   if (p->d != kD) return ECOKV_ERR_UNSUPPORTED;
   if (p->n > kMaxN) return ECOKV_ERR_UNSUPPORTED;
@@ -368,12 +381,12 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   f.S = S;
   f.lambda = lambda;
   f.dbg = dbg;
-  if ((st = winsor_check(*p, L)) != ECOKV_OK) return st;
+  if ((st = robust_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
   stage_event(1, s);
-  if ((st = winsor_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
+  if ((st = robust_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
   if (run_finalize(f, L.U, false, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   stage_event(2, s);
   return ECOKV_OK;
@@ -436,12 +449,12 @@ ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, cons
   FinalArgs f = final_args(*p, L, w);
   f.S = reinterpret_cast<float*>(w + L.sbuf);
   f.lambda = lambda;
-  if ((st = vnorm_check(*p, L)) != ECOKV_OK || (st = winsor_check(*p, L)) != ECOKV_OK) return st;
+  if ((st = vnorm_check(*p, L)) != ECOKV_OK || (st = robust_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
   if ((st = vnorm_launch(*p, dtype, L, V, w, f, s)) != ECOKV_OK) return st;
-  if ((st = winsor_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
+  if ((st = robust_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
   stage_event(1, s);
   if (run_finalize(f, L.U, false, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   // 2. one top-h_kv (B - W) per layer over its heads' concatenated scores
@@ -505,12 +518,12 @@ static ecokv_status evict_impl(const ecokv_params* p, ecokv_dtype dtype, const v
       c.keep[l] = layer_budget[l] < p->n ? layer_budget[l] : p->n;
     }
   }
-  if ((st = vnorm_check(*p, L)) != ECOKV_OK || (st = winsor_check(*p, L)) != ECOKV_OK) return st;
+  if ((st = vnorm_check(*p, L)) != ECOKV_OK || (st = robust_check(*p, L)) != ECOKV_OK) return st;
   stage_event(0, s);
   st = tc ? run_tc_passes(*p, K, Qwin, w, s) : run_simt_passes(*p, dtype, K, Qwin, w, s);
   if (st != ECOKV_OK) return st;
   if ((st = vnorm_launch(*p, dtype, L, V, w, f, s)) != ECOKV_OK) return st;
-  if ((st = winsor_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
+  if ((st = robust_launch(*p, L, w, f, s)) != ECOKV_OK) return st;
   stage_event(1, s);
   if (run_finalize(f, L.U, true, s) != ECOKV_OK) return ECOKV_ERR_CUDA;
   stage_event(2, s);

@@ -104,6 +104,12 @@ struct FinalArgs {
   // bounds of d_E, at wlo[4 u] and whi[4 u]; null for the plain min-max
   const unsigned* wlo;
   const unsigned* whi;
+  // MAD scaling: the order-preserving keys of the two middle order
+  // statistics of d_E at mad[4 u] and mad[4 (n_units + u)] (their mean is
+  // the median), and of |d_E - median| at mad[4 (2 n_units + u)] and
+  // mad[4 (3 n_units + u)] (their mean is the MAD); null otherwise
+  const unsigned* mad;
+  int n_units;
   // per-layer budgets (PyramidKV schedule): with n_lb > 0 the heads of layer
   // l keep lb[l] rows (window included) in slots of stride n_keep
   int h_kv, n_lb;
@@ -152,11 +158,12 @@ cudaError_t launch_value_norms(const void* V, ecokv_dtype dt, int U, int N, int 
 bool cluster_finalize_fits(int Tv);
 // k largest of each layer's T scores, ascending positions (layer_select.cu)
 size_t layer_select_scratch_bytes(int n_layers, int T);
-// the k1-th and the k2-th largest of each row's T values (their
-// order-preserving keys at state[4 row] and state[4 (rows + row)]);
-// hist: 2 * rows * 2048 unsigned, state: 2 * rows * 4 unsigned
-cudaError_t launch_row_kth2(const float* S, int rows, int T, int k1, int k2, unsigned* hist, unsigned* state,
-                            cudaStream_t s);
+// the order-preserving keys of the ka-th and kb-th largest of each row's
+// T <= 32768 values at out[4 row] and out[4 (rows + row)]; with mad also
+// those of |x - m| (m the mean of the first two) at out[4 (2 rows + row)]
+// and out[4 (3 rows + row)] (order_stats.cu)
+cudaError_t launch_order_stats(const float* x, int rows, int T, int ka, int kb, bool mad, unsigned* out,
+                               cudaStream_t s);
 cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int32_t* chosen, void* scratch,
                                 cudaStream_t s);
 // One thread-block cluster per unit: scores, and the top-k when f.idx is set

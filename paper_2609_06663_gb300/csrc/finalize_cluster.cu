@@ -68,15 +68,16 @@ struct ClusterSmem {
   unsigned hall[2][Shape<kJ>::kMaxCluster][256];
   float ext_all[Shape<kJ>::kMaxCluster][2];
   double simp_all[Shape<kJ>::kMaxCluster];  // value-norm importance: every rank's sum of S_imp
-  double wsum_all[Shape<kJ>::kMaxCluster];  // winsorised min-max: every rank's sum of the clipped d_E
+  double wsum_all[Shape<kJ>::kMaxCluster];  // winsorised min-max / MAD scaling: every rank's sum of s_E terms
   int cnt_all[Shape<kJ>::kMaxCluster][2];
   float red[kCWarps][8];  // per-warp partials
   float edge[32];         // pooling edge values
   float sc[8];            // broadcast scalars
   double dsc[2];          // sums behind the means of S_imp and of S_div
   double dred[kCWarps];   // per-warp sums of S_imp (value-norm importance)
-  double dredw[kCWarps];  // per-warp sums of the clipped d_E (winsorised min-max)
+  double dredw[kCWarps];  // per-warp sums of the clipped d_E (winsorised min-max) or of s_E (MAD scaling)
   float wmax;             // winsorised min-max: the upper clip bound
+  float mmed, minv;       // MAD scaling: the median of d_E and 1 / (MAD + eps)
   unsigned wsum[kCWarps];
   int wscan[kCWarps][2];  // per-warp counts above / equal to the threshold
   int shi[4];
@@ -91,9 +92,10 @@ __device__ __forceinline__ float sdiv_rcp(float dE, float c, float mnE, float in
   return __fadd_rn(__fmul_rn(alpha, sE), __fmul_rn(__fsub_rn(1.f, alpha), sC));
 }
 
-// The float an order-preserving key stands for (the inverse of ordered_key).
-__device__ __forceinline__ float key_float(unsigned k) {
-  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+// MAD scaling of a distance (the robust form of Eq. 2): the logistic
+// function of (d_E - median) / (MAD + eps), the divisor as a reciprocal.
+__device__ __forceinline__ float mad_logistic(float dE, float med, float inv) {
+  return 1.f / (1.f + expf(-__fmul_rn(__fsub_rn(dE, med), inv)));
 }
 
 // Store v into the same object of every CTA of the cluster (its own included).
@@ -105,8 +107,8 @@ __device__ __forceinline__ void push_all(cg::cluster_group& cl, T* obj, T v, int
 }
 
 // kMode: 0 = scores, 1 = scores and top-k, 2 = top-k of given scores (f.S).
-// kVar: the value-norm importance and winsorised min-max variants are compiled
-// in (their code is left out of the default kernel, whose register budget it
+// kVar: the value-norm importance, winsorised min-max and MAD scaling
+// variants are compiled in (their code is left out of the default kernel, whose register budget it
 // would cost).
 template <int kMode, int kJ, bool kVar>
 __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArgs f) {
@@ -273,6 +275,17 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       sm.sc[0] = s_all;
       sm.sc[1] = mnE;
       sm.sc[2] = __fadd_rn(__fsub_rn(mxE, mnE), f.eps);
+      if (kVar && f.mad != nullptr) {
+        // MAD scaling: the sweep maps d_E to s_E itself, so the affine map
+        // that follows it is the identity
+        const int nu = f.n_units;
+        const float lo2 = key_float(f.mad[4 * u]), hi2 = key_float(f.mad[4 * (nu + u)]);
+        const float dlo = key_float(f.mad[4 * (2 * nu + u)]), dhi = key_float(f.mad[4 * (3 * nu + u)]);
+        sm.mmed = __fmul_rn(0.5f, __fadd_rn(lo2, hi2));
+        sm.minv = 1.f / __fadd_rn(__fmul_rn(0.5f, __fadd_rn(dlo, dhi)), f.eps);
+        sm.sc[1] = 0.f;
+        sm.sc[2] = 1.f;
+      }
       sm.sc[3] = s_de;
       sm.sc[4] = s_c;
       sm.sc[5] = s_raw;
@@ -293,14 +306,15 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         if (i < Tv) sm.raw[pad_idx(i - lo + kHalo)] = __ldg(vnu + i);
       }
       __syncthreads();
-      double ps = 0.0;
+      float psf = 0.f;  // a thread's at most 32 terms in single precision, the reductions in double
   #pragma unroll
       for (int c = 0; c < kJ; ++c)
         if (c < nv) {
           const float si = __fmul_rn(__uint_as_float(key[c]), sm.raw[pad_idx(q0 + c)]);
           key[c] = __float_as_uint(si);
-          ps += (double)si;
+          psf = __fadd_rn(psf, si);
         }
+      double ps = (double)psf;
   #pragma unroll
       for (int o = 16; o > 0; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
       if (lane == 0) sm.dred[warp] = ps;
@@ -349,8 +363,11 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
     //    cluster
     float mnD = INFINITY, mxD = -INFINITY;
     const bool wins = kVar && f.wlo != nullptr;
-    const float wmax = sm.wmax;
-    double wsum = 0.0;  // winsorised min-max: this thread's sum of clipped d_E
+    const bool madv = kVar && f.mad != nullptr;
+    const float wmax = sm.wmax, mmed = sm.mmed, minv = sm.minv;
+    // this thread's sum of the clipped d_E (winsorised min-max) or of s_E (MAD
+    // scaling): at most 32 terms in single precision, the reductions in double
+    float wsumf = 0.f;
     {
       const float* dEu = f.dE + (size_t)u * Tv;
       const float* cvu = f.cosv + (size_t)u * Tv;
@@ -376,7 +393,10 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
               if (i + r < Tv) {
                 if (wins) {
                   e[r] = fminf(fmaxf(e[r], mnE), wmax);
-                  wsum += (double)e[r];
+                  wsumf = __fadd_rn(wsumf, e[r]);
+                } else if (madv) {
+                  e[r] = mad_logistic(e[r], mmed, minv);
+                  wsumf = __fadd_rn(wsumf, e[r]);
                 }
                 const float sd = sdiv_rcp(e[r], cs[r], mnE, invE, f.alpha, mix);
                 sm.raw[pad_idx(i + r - lo + kHalo)] = sd;
@@ -393,7 +413,10 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
             float e = __ldg(dEu + i);
             if (wins) {
               e = fminf(fmaxf(e, mnE), wmax);
-              wsum += (double)e;
+              wsumf = __fadd_rn(wsumf, e);
+            } else if (madv) {
+              e = mad_logistic(e, mmed, minv);
+              wsumf = __fadd_rn(wsumf, e);
             }
             const float sd = sdiv_rcp(e, __ldg(cvu + i), mnE, invE, f.alpha, mix);
             sm.raw[pad_idx(i - lo + kHalo)] = sd;
@@ -403,7 +426,8 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         }
       }
     }
-    if (wins) {
+    if (wins || madv) {
+      double wsum = (double)wsumf;
   #pragma unroll
       for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
       if (lane == 0) sm.dredw[warp] = wsum;
@@ -432,7 +456,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         for (int w = 0; w < kCWarps; ++w) cs += sm.dred[w];
         push_all<kMaxC>(cl, &sm.simp_all[rank], cs, C);
       }
-      if (wins) {
+      if (wins || madv) {
         double cs = 0.0;
         for (int w = 0; w < kCWarps; ++w) cs += sm.dredw[w];
         push_all<kMaxC>(cl, &sm.wsum_all[rank], cs, C);
@@ -448,7 +472,7 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
       const float denD = __fadd_rn(__fsub_rn(a1, a0), f.eps);
       // mean(S_imp) / mean(Sbar) with Sbar = (S_div - a0) / denD
       double dsc1 = sm.dsc[1];  // Tv * mean(S_div)
-      if (wins) {  // s_E from the clipped distances: their sum replaces the sum of d_E
+      if (wins || madv) {  // s_E from the clipped distances (or s_E itself): that sum replaces the sum of d_E
         double sum_clip = 0.0;
         for (int r = 0; r < C; ++r) sum_clip += sm.wsum_all[r];
         const double T = (double)Tv, s_c = (double)sm.sc[4];
@@ -501,7 +525,8 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
         dbg[Tv + i] = __fmul_rn(acc, inv_pool);
         dbg[2 * Tv + i] = e;
         dbg[3 * Tv + i] = cs;
-        dbg[4 * Tv + i] = sdiv_rcp(wins ? fminf(fmaxf(e, mnE), wmax) : e, cs, mnE, invE, f.alpha, mix);
+        const float ev = wins ? fminf(fmaxf(e, mnE), wmax) : madv ? mad_logistic(e, mmed, minv) : e;
+        dbg[4 * Tv + i] = sdiv_rcp(ev, cs, mnE, invE, f.alpha, mix);
       }
     }
     if (f.S != nullptr) {
@@ -714,7 +739,7 @@ cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cud
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  const bool var = f.vnorm != nullptr || f.wlo != nullptr;
+  const bool var = f.vnorm != nullptr || f.wlo != nullptr || f.mad != nullptr;
   if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ, false>, f);
   if (f.idx == nullptr)
     return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ, true>, f)

@@ -224,6 +224,11 @@ __device__ __forceinline__ unsigned ordered_key(float f) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
+// The float an order-preserving key stands for (the inverse of ordered_key).
+__device__ __forceinline__ float key_float(unsigned k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 // Top-k of S[0..Tv) by (value desc, position asc), written in ascending
 // position to out[0..k).  hist: 256 unsigned, shi: >= 64 ints (shared).
 template <class Sync>

@@ -29,7 +29,6 @@ constexpr int kLsWarpSpan = kLsSpan / kLsWarps;  // contiguous scores a warp emi
 struct LsArgs {
   const float* S;     // [L][T]
   int T, k, nblk;
-  int k2, rows;       // a second selection (grid z = 1): k2-th largest, its histograms and state after the first's
   unsigned* ghist;    // [L][kLsMaxBins], zero before the first digit
   unsigned* state;    // [L][4]: prefix, mask, remaining count at the threshold (zero before the first digit)
   int* cnt;           // [L][nblk][2]: a block's scores above / equal to the threshold
@@ -51,8 +50,7 @@ __global__ void __launch_bounds__(kLsThreads) ls_hist(LsArgs a, int shift) {
   ls_wait();
   __syncthreads();
   const float* S = a.S + (size_t)l * a.T;
-  const size_t z = blockIdx.z;  // which selection
-  const unsigned* st = a.state + 4 * (z * a.rows + l);
+  const unsigned* st = a.state + 4 * l;
   const unsigned prefix = st[0], mask = st[1];
 #pragma unroll 4
   for (int j = 0; j < kLsPer; ++j) {
@@ -69,7 +67,7 @@ __global__ void __launch_bounds__(kLsThreads) ls_hist(LsArgs a, int shift) {
   }
   __syncthreads();
   for (int b = tid; b < kBins; b += kLsThreads)
-    if (hist[b]) atomicAdd(a.ghist + (z * a.rows + l) * kLsMaxBins + b, hist[b]);
+    if (hist[b]) atomicAdd(a.ghist + (size_t)l * kLsMaxBins + b, hist[b]);
 }
 
 template <int kBits>
@@ -78,10 +76,9 @@ __global__ void __launch_bounds__(256) ls_digit(LsArgs a, int shift, int first) 
   const int l = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   __shared__ unsigned wsum[8];
   ls_wait();
-  const size_t z = blockIdx.z;  // which selection
-  unsigned* st = a.state + 4 * (z * a.rows + l);
-  unsigned* gh = a.ghist + (z * a.rows + l) * kLsMaxBins + tid * kPer;
-  const unsigned rem = first ? (unsigned)(z ? a.k2 : a.k) : st[2];
+  unsigned* st = a.state + 4 * l;
+  unsigned* gh = a.ghist + (size_t)l * kLsMaxBins + tid * kPer;
+  const unsigned rem = first ? (unsigned)a.k : st[2];
   unsigned h[kPer], tot = 0u;
 #pragma unroll
   for (int q = 0; q < kPer; ++q) {
@@ -248,7 +245,6 @@ cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int3
   a.state = a.ghist + (size_t)n_layers * kLsMaxBins;
   a.cnt = reinterpret_cast<int*>(a.state + (size_t)n_layers * 4);
   a.chosen = chosen;
-  a.rows = n_layers;
   cudaError_t e = cudaMemsetAsync(scratch, 0, (size_t)n_layers * (kLsMaxBins + 4) * 4, s);
   if (e != cudaSuccess) return e;
   const dim3 grid(a.nblk, n_layers), blk(kLsThreads);
@@ -260,31 +256,6 @@ cudaError_t launch_layer_select(const float* S, int n_layers, int T, int k, int3
       (e = launch_dependent(ls_digit<10>, dim3(n_layers), dim3(256), s, a, 0, 0)) != cudaSuccess ||
       (e = launch_dependent(ls_count, grid, blk, s, a)) != cudaSuccess ||
       (e = launch_dependent(ls_emit, grid, blk, s, a)) != cudaSuccess)
-    return e;
-  return cudaSuccess;
-}
-
-cudaError_t launch_row_kth2(const float* S, int rows, int T, int k1, int k2, unsigned* hist, unsigned* state,
-                            cudaStream_t s) {
-  if (rows <= 0 || T <= 0 || k1 < 1 || k1 > T || k2 < 1 || k2 > T) return cudaErrorInvalidValue;
-  LsArgs a{};
-  a.S = S;
-  a.T = T;
-  a.k = k1;
-  a.k2 = k2;
-  a.rows = rows;
-  a.nblk = (T + kLsSpan - 1) / kLsSpan;
-  a.ghist = hist;
-  a.state = state;
-  cudaError_t e = cudaMemsetAsync(hist, 0, (size_t)2 * rows * kLsMaxBins * 4, s);
-  if (e != cudaSuccess || (e = cudaMemsetAsync(state, 0, (size_t)2 * rows * 4 * 4, s)) != cudaSuccess) return e;
-  const dim3 grid(a.nblk, rows, 2), dgrid(rows, 1, 2), blk(kLsThreads);
-  if ((e = launch_dependent(ls_hist<11>, grid, blk, s, a, 21)) != cudaSuccess ||
-      (e = launch_dependent(ls_digit<11>, dgrid, dim3(256), s, a, 21, 1)) != cudaSuccess ||
-      (e = launch_dependent(ls_hist<11>, grid, blk, s, a, 10)) != cudaSuccess ||
-      (e = launch_dependent(ls_digit<11>, dgrid, dim3(256), s, a, 10, 0)) != cudaSuccess ||
-      (e = launch_dependent(ls_hist<10>, grid, blk, s, a, 0)) != cudaSuccess ||
-      (e = launch_dependent(ls_digit<10>, dgrid, dim3(256), s, a, 0, 0)) != cudaSuccess)
     return e;
   return cudaSuccess;
 }

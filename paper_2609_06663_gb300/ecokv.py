@@ -19,6 +19,7 @@ ECOKV_FLAG_VNORM_IMP = 0x4
 ECOKV_FLAG_CENTROID_NONWIN = 0x8
 ECOKV_FLAG_WINSOR_1 = 0x10
 ECOKV_FLAG_WINSOR_5 = 0x20
+ECOKV_FLAG_MAD = 0x40
 ECOKV_FLAG_FORCE_SIMT = 0x100
 ECOKV_NOALLOC_SCRATCH_BYTES = 16 << 20   # fixed scratch of ecokv_evict_noalloc, per device
 ECOKV_OK, ECOKV_ERR_INVALID_ARG, ECOKV_ERR_UNSUPPORTED, ECOKV_ERR_WORKSPACE = 0, 1, 2, 3

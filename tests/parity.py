@@ -16,7 +16,8 @@ def oracle_params(p, **over) -> O.Params:
     kw = {k: getattr(p, k) for k in ("n_layers", "h_kv", "h_q", "n", "d", "window", "budget", "pool_kernel",
                                       "alpha", "beta", "tau", "eps", "flags", "lambda_override")}
     kw["flags"] = kw["flags"] & (O.FLAG_SC_MIXKV_SIGN | O.FLAG_LAMBDA_OVERRIDE | O.FLAG_VNORM_IMP |
-                                 O.FLAG_CENTROID_NONWIN | O.FLAG_WINSOR_1 | O.FLAG_WINSOR_5)  # path flags mean nothing here
+                                 O.FLAG_CENTROID_NONWIN | O.FLAG_WINSOR_1 | O.FLAG_WINSOR_5 |
+                                 O.FLAG_MAD)  # path flags mean nothing here
     kw.update(over)
     return O.Params(**kw)
 

@@ -131,6 +131,12 @@ def test_adaptive_entry_rejects_bad_arguments(lib):
     # both winsorising levels at once
     p.flags = E.ECOKV_FLAG_WINSOR_1 | E.ECOKV_FLAG_WINSOR_5
     assert E.ecokv_check_params(p) == 1
+    # MAD scaling with a winsorising level
+    for wf in (E.ECOKV_FLAG_WINSOR_1, E.ECOKV_FLAG_WINSOR_5):
+        p.flags = E.ECOKV_FLAG_MAD | wf
+        assert E.ecokv_check_params(p) == 1
+    p.flags = E.ECOKV_FLAG_MAD
+    assert E.ecokv_check_params(p) == 0
 
 
 def test_status_strings(lib):

@@ -257,3 +257,21 @@ def test_winsorised_minmax(w, flags):
 
 def test_winsorised_minmax_c2_two_layers():
     run_and_compare(CONFIGS["c2"], layers=range(10, 12), flags=E.ECOKV_FLAG_WINSOR_5)
+
+
+# MAD scaling of Eq. 2 (reading R21): both streaming paths, an odd and an even
+# candidate count, against the oracle (scores, lambda, the per-token terms,
+# selection, rows)
+@pytest.mark.parametrize("w,flags", [
+    (small_workload(5000, h_kv=2, group=4, window=8, budget=500, dtype="bf16", n_layers=2, clustered=True), 0),
+    (small_workload(20001, h_kv=2, group=4, window=8, budget=2000, dtype="bf16", clustered=True), 0),
+    (small_workload(5000, h_kv=2, group=4, window=8, budget=500, dtype="bf16", clustered=True),
+     E.ECOKV_FLAG_FORCE_SIMT),
+    (small_workload(3001, h_kv=2, group=1, window=8, budget=300, pool_kernel=7, dtype="f32"), 0),
+], ids=["bf16_tc_even", "bf16_wide_odd", "bf16_simt", "f32_simt_odd"])
+def test_mad_scaling(w, flags):
+    run_and_compare(w, flags=flags | E.ECOKV_FLAG_MAD)
+
+
+def test_mad_scaling_c2_two_layers():
+    run_and_compare(CONFIGS["c2"], layers=range(6, 8), flags=E.ECOKV_FLAG_MAD)
