@@ -133,6 +133,13 @@ def test_sweep_points(n, window):
     run_and_compare(sweep_workload(n, window))
 
 
+def test_sweep_largest_point_sampled_heads():
+    # the sweep's longest layer (131072 tokens, W = 16: g W = 64 rows on the
+    # tensor cores; 131056 candidates, so the one-CTA finalize), every head
+    # scored in one call, two heads against the oracle
+    run_and_compare(sweep_workload(131072, 16), units=[(0, 0), (0, 5)])
+
+
 def test_identical_keys_all_ties():
     # Every key equal: d_E = 0 and r_E = r_C = 1, so lambda = 1 and S_div is
     # constant; Sbar vanishes and S = 0 for every candidate in exact
