@@ -282,3 +282,40 @@ def test_mad_scaling(w, flags):
 
 def test_mad_scaling_c2_two_layers():
     run_and_compare(CONFIGS["c2"], layers=range(6, 8), flags=E.ECOKV_FLAG_MAD)
+
+
+# the order statistics behind the robust forms of Eq. 2 are exact: S_div
+# recomputed in double from the GPU's own d_E and cosines, with numpy's order
+# statistics of those single-precision distances (the median and MAD formed
+# in single precision, as the kernels form them), agrees to rounding; a rank
+# off by one moves s_E by ~1e-4
+@pytest.mark.parametrize("flags", [E.ECOKV_FLAG_WINSOR_5, E.ECOKV_FLAG_WINSOR_1, E.ECOKV_FLAG_MAD],
+                         ids=["winsor5", "winsor1", "mad"])
+@pytest.mark.parametrize("n", [5000, 20001, 32768])
+def test_robust_order_statistics_exact(flags, n):
+    w = small_workload(n, h_kv=2, group=4, window=8, budget=n // 10, dtype="bf16", clustered=True, seed=3)
+    K, V, Q = make_inputs(w)
+    p = params_of(w, flags=flags)
+    ws = E.alloc_workspace(p, DEV)
+    _, _, dbg = E.score(p, K.to(DEV), Q.to(DEV), ws=ws, dbg=True)
+    torch.cuda.synchronize()
+    assert E.ecokv_device_status(ws) == 0
+    dbg = dbg.cpu().numpy()
+    for h in range(w.h_kv):
+        dE = dbg[0, h, 2].astype(np.float32)
+        c = dbg[0, h, 3].astype(np.float64)
+        T = dE.size
+        srt = np.sort(dE)
+        if flags & E.ECOKV_FLAG_MAD:
+            half = np.float32(0.5)
+            med = half * (srt[(T - 1) // 2] + srt[T // 2])
+            dev = np.sort(np.abs(dE - med))
+            mad = half * (dev[(T - 1) // 2] + dev[T // 2])
+            sE = 1.0 / (1.0 + np.exp(-(dE.astype(np.float64) - float(med)) / (float(mad) + float(p.eps))))
+        else:
+            q = 0.01 if flags & E.ECOKV_FLAG_WINSOR_1 else 0.05
+            lo, hi = float(srt[int(np.floor(q * (T - 1)))]), float(srt[int(np.ceil((1 - q) * (T - 1)))])
+            sE = (np.clip(dE.astype(np.float64), lo, hi) - lo) / (hi - lo + float(p.eps))
+        sdiv = float(p.alpha) * sE + (1.0 - float(p.alpha)) * (1.0 - c) / 2.0
+        err = np.abs(dbg[0, h, 4].astype(np.float64) - sdiv).max()
+        assert err <= 2e-6, f"n={n} head {h}: S_div differs by {err:.2e} from the exact order statistics"
