@@ -13,6 +13,8 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "ecokv_internal.cuh"
 #include "tc_pass.cuh"
 
@@ -99,15 +101,15 @@ static int tc_chunk_keys(const ecokv_params& p) { return 128 * tc_tiles(p); }
 
 // SMs of the current device (cached per device).
 static int num_sms() {
-  static int cached[64] = {0};
+  static std::atomic<int> cached[64];  // a racing thread repeats the query
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
-  if (cached[dev] == 0) {
+  if (cached[dev].load() == 0) {
     int n = 0;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
-    cached[dev] = n;
+    cached[dev].store(n);
   }
-  return cached[dev];
+  return cached[dev].load();
 }
 
 static int env_int(const char* name, int dflt, int lo, int hi) {

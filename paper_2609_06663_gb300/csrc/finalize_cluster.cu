@@ -34,6 +34,8 @@
 // (each CTA keeps every rank's contribution) followed by a cluster barrier,
 // so no CTA waits on a remote load.
 
+#include <atomic>
+
 #include <cooperative_groups.h>
 
 #include "finalize_select.cuh"
@@ -766,14 +768,14 @@ cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only,
   const int C32 = (Tv + Shape<32>::kCap - 1) / Shape<32>::kCap;
   const bool wide = C16 > 4;
   if (wide ? C32 > Shape<32>::kMaxCluster : C16 > Shape<16>::kMaxCluster) return cudaErrorNotSupported;
-  static bool attr_set[64] = {};
+  static std::atomic<bool> attr_set[64];  // a racing thread repeats the idempotent setup
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!attr_set[dev]) {
+  if (!attr_set[dev].load()) {
     if ((e = set_smem_attrs<16>()) != cudaSuccess || (e = set_smem_attrs<32>()) != cudaSuccess) return e;
-    attr_set[dev] = true;
+    attr_set[dev].store(true);
   }
   return wide ? launch_shape<32>(f, U, C32, select_only, s) : launch_shape<16>(f, U, C16, select_only, s);
 }

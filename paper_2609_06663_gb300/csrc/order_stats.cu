@@ -19,6 +19,8 @@
 // ranks (MAD: all four, the second pair over |d_E - median|) where a
 // grid-wide select needs a launch per digit.
 
+#include <atomic>
+
 #include "ecokv_internal.cuh"
 #include "finalize_select.cuh"
 
@@ -276,18 +278,18 @@ cudaError_t launch_order_stats(const float* x, int rows, int T, int ka, int kb, 
   cfg.blockDim = dim3(kOsThreads);
   cfg.dynamicSmemBytes = sizeof(OsSmem);
   cfg.stream = s;
-  static bool attr_set[64] = {};
+  static std::atomic<bool> attr_set[64];  // a racing thread repeats the idempotent setup
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!attr_set[dev]) {
+  if (!attr_set[dev].load()) {
     if ((e = cudaFuncSetAttribute(order_stats_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)sizeof(OsSmem))) != cudaSuccess ||
         (e = cudaFuncSetAttribute(order_stats_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)sizeof(OsSmem))) != cudaSuccess)
       return e;
-    attr_set[dev] = true;
+    attr_set[dev].store(true);
   }
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -44,6 +44,8 @@
 // copies and MMAs, frees TMEM and exits.
 
 #include <cuda.h>
+
+#include <atomic>
 #include <stddef.h>
 
 #include "finalize_select.cuh"
@@ -1041,14 +1043,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-int g_num_sms[64] = {0};
-bool g_attr_set[64][4] = {};
+// per-device host state; a racing thread repeats the idempotent setup
+std::atomic<int> g_num_sms[64];
+std::atomic<bool> g_attr_set[64][4];
 
 template <int RH>
 cudaError_t launch_rh(const CUtensorMap& tm, const CUtensorMap& tq, const TcArgs& a, int dev, cudaStream_t st) {
   const size_t smem = sizeof(Smem<RH>) + 1024;
   const int rh_i = RH == 8 ? 0 : RH == 16 ? 1 : RH == 32 ? 2 : 3;
-  if (!g_attr_set[dev][rh_i]) {
+  if (!g_attr_set[dev][rh_i].load()) {
     // the warpgroups' register split needs the launch to give every thread
     // 65536 / kThreads registers; refuse to launch otherwise
     cudaFuncAttributes fa;
@@ -1057,9 +1060,9 @@ cudaError_t launch_rh(const CUtensorMap& tm, const CUtensorMap& tq, const TcArgs
     if (fa.numRegs * kThreads < 2 * 128 * (int)(kRegsEpi + kRegsOther)) return cudaErrorInvalidConfiguration;
     e = cudaFuncSetAttribute(tc_evict_kernel<RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    g_attr_set[dev][rh_i] = true;
+    g_attr_set[dev][rh_i].store(true);
   }
-  tc_evict_kernel<RH><<<g_num_sms[dev], kThreads, smem, st>>>(tm, tq, a);
+  tc_evict_kernel<RH><<<g_num_sms[dev].load(), kThreads, smem, st>>>(tm, tq, a);
   return cudaGetLastError();
 }
 
@@ -1068,16 +1071,19 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  if (fn == nullptr) {
+  static std::atomic<EncodeTiledFn> fn{nullptr};  // a racing thread repeats the lookup
+  EncodeTiledFn f = fn.load();
+  if (f == nullptr) {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
             cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
+        q == cudaDriverEntryPointSuccess) {
+      f = reinterpret_cast<EncodeTiledFn>(p);
+      fn.store(f);
+    }
   }
-  return fn;
+  return f;
 }
 
 }  // namespace
@@ -1096,9 +1102,11 @@ cudaError_t launch_tc(const void* K, const TcArgs& args, cudaStream_t st) {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (g_num_sms[dev] == 0) {
-    e = cudaDeviceGetAttribute(&g_num_sms[dev], cudaDevAttrMultiProcessorCount, dev);
+  if (g_num_sms[dev].load() == 0) {
+    int n = 0;
+    e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
+    g_num_sms[dev].store(n);
   }
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return cudaErrorNotSupported;
