@@ -57,6 +57,35 @@ def test_value_norm_importance(case):
 
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("flags", [
+    E.ECOKV_FLAG_VNORM_IMP | E.ECOKV_FLAG_MAD,
+    E.ECOKV_FLAG_VNORM_IMP | E.ECOKV_FLAG_WINSOR_1 | E.ECOKV_FLAG_CENTROID_NONWIN,
+    E.ECOKV_FLAG_MAD | E.ECOKV_FLAG_CENTROID_NONWIN | E.ECOKV_FLAG_SC_MIXKV_SIGN,
+], ids=["vnorm_mad", "vnorm_winsor1_nonwin", "mad_nonwin_mixsign"])
+@pytest.mark.parametrize("case", CASES[:2], ids=IDS[:2])
+def test_combined_variant_flags(case, flags):
+    # the variants compose: each flag changes an independent term of the score
+    w, units = case
+    K, V, Q = make_inputs(w)
+    p = params_of(w, flags)
+    idx, Ko, Vo, S, lam = E.evict(p, K.to(DEV), V.to(DEV), Q.to(DEV), want_scores=True)
+    torch.cuda.synchronize()
+    op = oracle_params(p)
+    assert op.flags == flags
+    units = [(l, h) for l in range(w.n_layers) for h in range(w.h_kv)]
+    ref = O.evict(K, V, Q, op, heads=units)
+    tol = TOL[w.dtype]
+    S_np = S.cpu().double().numpy()
+    for (l, h) in units:
+        r = ref[(l, h)]
+        what = f"{w.name} unit ({l},{h}) flags {flags:#x}"
+        assert score_error(S_np[l, h], r["S"]) <= tol, what
+        assert abs(float(lam[l, h]) - r["lam"]) <= tol, what
+        check_selection(idx[l, h].cpu().numpy(), r, op, tol, what)
+        check_rows(V[l, h].to(DEV), idx[l, h], Vo[l, h], what)
+
+
+@pytest.mark.gpu
 def test_value_norm_flag_changes_the_scores_and_is_refused_without_values():
     w = CASES[0][0]
     K, V, Q = make_inputs(w, device=DEV)
