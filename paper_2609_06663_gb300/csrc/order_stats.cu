@@ -46,15 +46,16 @@ struct OsSmem {
 // Stage index of row position q (thread q / kOsPer's key q % kOsPer).
 __device__ __forceinline__ int os_pad(int q) { return q + (q / kOsPer) * kOsPad; }
 
-// Row u of x into the stage as keys, |x - m| with kDev.
+// The key of a value: of v, or with kDev of |v - m|.
 template <bool kDev>
 __device__ __forceinline__ unsigned os_key(float v, float m) {
   return ordered_key(kDev ? fabsf(__fsub_rn(v, m)) : v);
 }
+
+// The row's T values at xr into the stage as keys, coalesced; a thread
+// issues all of its loads before its first store.
 template <bool kDev>
 __device__ __forceinline__ void os_stage(const float* xr, int T, float m, OsSmem& sm, int tid) {
-  // every load of a thread issued before its first store (the row comes
-  // from L2 or DRAM: one round trip, not one per load)
   constexpr int kV = kOsPer / 4;  // 16-byte loads per thread
   if ((reinterpret_cast<uintptr_t>(xr) & 15u) == 0) {
     const int n4 = T >> 2;
