@@ -166,6 +166,28 @@ def test_euclid_redundancy_closed_forms():
     assert vals[0] == 1.0 and all(a > b for a, b in zip(vals, vals[1:])) and vals[-1] > 0
 
 
+def test_mean_distance_below_rms_distance():
+    # Appendix C's standard-deviation alternative: D_std = sqrt(mean ||k_i -
+    # kbar||^2), here by the variance identity sqrt(mean ||k||^2 - ||kbar||^2);
+    # Jensen gives D_E <= D_std, with equality when every key is equally far
+    # from the centroid
+    r = rng(30)
+    n, d = 40, 16
+    K, _ = aniso(r, n, d)
+    out = O.score_head(K, r.standard_normal((1, 2, d)), params(n, d, window=2, budget=10))
+    kbar = K.mean(axis=0)
+    d_std = math.sqrt((K * K).sum(axis=1).mean() - kbar @ kbar)
+    assert out["D_E"] < d_std * (1 - 1e-3)                  # spread distances: strict
+    # keys on a sphere about their centroid (pairs +-v_i): every distance equal
+    V = r.standard_normal((n // 2, d))
+    V *= 3.0 / np.linalg.norm(V, axis=1, keepdims=True)
+    S2 = np.vstack([V, -V]) + 5.0
+    out2 = O.score_head(S2, r.standard_normal((1, 2, d)), params(n, d, window=2, budget=10))
+    c2 = S2.mean(axis=0)
+    d_std2 = math.sqrt((S2 * S2).sum(axis=1).mean() - c2 @ c2)
+    assert out2["D_E"] == pytest.approx(3.0, rel=1e-12) and d_std2 == pytest.approx(3.0, rel=1e-10)
+
+
 def test_minmax_range_and_order():
     x = rng(8).random(50) * 7 - 3
     s = O.minmax(x, 1e-6)
