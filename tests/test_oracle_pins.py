@@ -532,6 +532,11 @@ def test_mad_scaling_closed_forms():
     assert t[37] == pytest.approx(0.3775406687981454, rel=1e-14)     # logistic(-0.5)
     # eps enters the denominator
     assert O.mad_scale(x, 25.0)[100] == pytest.approx(0.7310585786300049, rel=1e-14)
+    # the smallest heads: one candidate is its own median (s = 1/2); two have
+    # their mean as median and half their gap as MAD (s = logistic(-1), logistic(1))
+    assert O.mad_scale(np.array([7.25]), 1e-6).tolist() == [0.5]
+    two = O.mad_scale(np.array([3.0, 11.0]), 0.0)
+    assert two[0] == pytest.approx(0.2689414213699951, rel=1e-14) and two[1] == pytest.approx(0.7310585786300049, rel=1e-14)
 
 
 def test_mad_scaling_invariances_and_outlier():
