@@ -86,6 +86,12 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
                                              a WINSOR flag (ECOKV_ERR_INVALID_ARG); heads of up to 32768
                                              candidates, else ECOKV_ERR_UNSUPPORTED */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
+#define ECOKV_FLAG_TEST_STALL      0x80000000u /* fault injection for tests of the bounded waits: the statistics of
+                                             the first unit (layer 0, KV head 0) are never complete, so pass 2
+                                             of that unit waits until timeout_us runs out; the call then records
+                                             ECOKV_ERR_TIMEOUT in the workspace's status word and its outputs
+                                             are unspecified.  Tensor-core path only (bf16, n >= 128), else
+                                             ECOKV_ERR_UNSUPPORTED */
 
 typedef struct {
   int32_t n_layers;    /* L >= 1 layers in one call                              */
@@ -103,11 +109,23 @@ typedef struct {
   float eps;           /* Eq. 2 min-max stabiliser, > 0 (1e-6)                     */
   uint32_t flags;      /* ECOKV_FLAG_* bits                                        */
   float lambda_override; /* lambda for every head when ECOKV_FLAG_LAMBDA_OVERRIDE  */
+  /* Schedule of the streaming kernel (bf16 tensor-core path); 0 selects the
+   * built-in default.  Results are deterministic for any setting, but the
+   * grouping of floating-point partial sums follows the schedule (and the
+   * device's SM count), so scores may differ in their last bits between
+   * settings (within the tolerances).  ecokv_workspace_size depends on
+   * sched_wave. */
+  int32_t sched_wave;    /* heads (layer, KV head) per wave of the schedule (default: all heads, i.e. pass 1
+                            of every head before any pass 2) */
+  int32_t sched_lag;     /* waves between a wave's first and second read of its keys (default 1) */
+  uint32_t timeout_us;   /* limit of every bounded device-side wait, microseconds (0 = 2 s); a wait that
+                            runs out records ECOKV_ERR_TIMEOUT in the status word */
 } ecokv_params;
 
 /* Fill *p with the paper's defaults (Appendix A.3): alpha 0.8, beta 0.6,
- * tau sqrt(d), eps 1e-6, pool_kernel 5, window 4, flags 0.  Shape fields are
- * zeroed and must be set by the caller. */
+ * tau sqrt(d), eps 1e-6, pool_kernel 5, window 4, flags 0, the default
+ * schedule and wait limit.  Shape fields are zeroed and must be set by the
+ * caller. */
 void ecokv_params_default(ecokv_params* p);
 
 /* Validate a parameter block.  Returns ECOKV_OK, ECOKV_ERR_INVALID_ARG (an
@@ -202,9 +220,13 @@ ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, cons
  * library's module on first use.  Nothing is allocated by the call: no
  * cudaMalloc, no allocating library routine.
  *   Arguments as for ecokv_evict, minus ws / ws_bytes, plus
- *   dev_status : optional (NULL to skip) device pointer, 4-byte aligned; in
- *                stream order after the pass it receives the call's device-side
- *                status (0, ECOKV_ERR_TIMEOUT or ECOKV_ERR_DEVICE_INDEX).
+ *   dev_status : optional device pointer, 4-byte aligned; in stream order
+ *                after the pass it receives the call's device-side status (0,
+ *                ECOKV_ERR_TIMEOUT or ECOKV_ERR_DEVICE_INDEX).  The scratch's
+ *                status word is cleared at the end of every call, so with
+ *                dev_status NULL a device-side error of the call is discarded
+ *                and nothing reports it (ecokv_device_status cannot reach the
+ *                scratch); pass a pointer wherever such errors matter.
  * Errors: everything ecokv_evict returns; ECOKV_ERR_WORKSPACE when the
  * workspace *p needs (ecokv_workspace_size) exceeds
  * ECOKV_NOALLOC_SCRATCH_BYTES, checked before anything is launched;
@@ -242,7 +264,9 @@ ecokv_status ecokv_evict_noalloc(const ecokv_params* p, ecokv_dtype dtype, const
  * link only for the kept rows; idx is copied back at the end.  Per call the
  * host link carries |K| + |Qwin| + B/n of |V| inbound and |K_out| + |V_out| +
  * |idx| outbound, against |K| + |V| + |Qwin| inbound for ecokv_evict on
- * copied inputs.  Returns after enqueueing; the outputs are valid once
+ * copied inputs.  Exception: with ECOKV_FLAG_VNORM_IMP the value norms are
+ * read from every row of V in host memory, so all of V crosses the link
+ * once more (|K| + |V| + |Qwin| + B/n of |V| inbound).  Returns after enqueueing; the outputs are valid once
  * `stream` has reached that point.  Scores are not returned (use
  * ecokv_score on device copies for them). */
 size_t ecokv_workspace_size_host(const ecokv_params* p, ecokv_dtype dtype);

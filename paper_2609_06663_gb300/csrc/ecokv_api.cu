@@ -22,30 +22,27 @@ namespace ecokv {
 
 static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
+Layout make_layout(const ecokv_params& p, int nrec) {
   Layout L{};
   L.U = p.n_layers * p.h_kv;
   L.R = (p.h_q / p.h_kv) * p.window;
   L.N = p.n;
   L.W = p.window;
   L.Tv = p.n - p.window;
-  L.chunk = chunk;
-  L.nchunks = (p.n + chunk - 1) / chunk;
-  L.p2slots = p2slots;
+  L.nchunks = nrec;
   L.p1_stride = 2 * ((L.R + 3) & ~3) + 2 * kD;
   L.ustat_stride = (ustat_lse() + L.R + 3) & ~3;
   const size_t U = (size_t)L.U;
   size_t off = 0;
   L.status = off;  off += 256;
-  L.sync = off;    L.sync_bytes = (4 + 4 * U) * 4;  off += align256(L.sync_bytes);
+  L.sync = off;    L.sync_bytes = (4 + 2 * U) * 4;  off += align256(L.sync_bytes);
   L.p1part = off;  off += align256(U * L.nchunks * L.p1_stride * 4);
   L.ustat = off;   off += align256(U * L.ustat_stride * 4);
-  L.p2part = off;  off += align256(U * L.nchunks * L.p2slots * kP2Stride * 4);
+  L.p2part = off;  off += align256(U * L.nchunks * kP2Stride * 4);
   L.simp = off;    off += align256(U * L.Tv * 4);
   L.dE = off;      off += align256(U * L.Tv * 4);
   L.cosv = off;    off += align256(U * L.Tv * 4);
   L.sbuf = off;    off += align256(U * L.Tv * 4);
-  L.norm2 = off;   off += align256(U * (size_t)L.N * 4);
   const size_t n_keep = (size_t)(p.budget < p.n ? p.budget : p.n);
   L.chosen = off;  off += align256(U * n_keep * 4);
   L.src = off;     off += align256(U * n_keep * 4);
@@ -58,8 +55,11 @@ Layout make_layout(const ecokv_params& p, int chunk, int p2slots) {
 
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+static int simt_records(const ecokv_params& p) { return (p.n + kChunk - 1) / kChunk; }
+static int tc_records(const ecokv_params& p);
+
 static size_t workspace_bytes(const ecokv_params& p) {
-  const size_t a = make_layout(p, kChunk).total, b = make_layout(p, kTcChunk, kTcP2Parts).total;
+  const size_t a = make_layout(p, simt_records(p)).total, b = make_layout(p, tc_records(p)).total;
   return a > b ? a : b;
 }
 
@@ -75,8 +75,6 @@ static bool use_tensor_path(const ecokv_params& p, ecokv_dtype dt) {
   return tc_rows_half((p.h_q / p.h_kv) * p.window) > 0;
 }
 
-static int env_int(const char* name, int dflt, int lo, int hi);
-
 // Stage events of this host thread (ecokv_set_stage_events), recorded on the
 // call's stream between its launches when set.
 thread_local cudaEvent_t g_stage_ev[4] = {nullptr, nullptr, nullptr, nullptr};
@@ -85,19 +83,27 @@ static void stage_event(int i, cudaStream_t s) {
   if (g_stage_ev[i] != nullptr) cudaEventRecord(g_stage_ev[i], s);
 }
 
-// Tiles of 128 keys per tensor-core pass item: the largest power of two up
-// to 64 that still leaves at least two items per SM (152 SMs) in each
-// pass, so that the persistent grid stays busy to its end while the per-item
-// costs (statistics, partial sums, scheduling) stay few.  ECOKV_TC_TILES
-// overrides it for tuning.
-static int tc_tiles(const ecokv_params& p) {
-  constexpr long long kItemsWanted = 2LL * 152;
-  int t = kTcMaxTiles;
+// Static schedule of the tensor-core kernel.  Units (heads) form waves
+// (ecokv_params.sched_wave heads each; 0 = one wave of every unit), each wave
+// cut into one slice per SM; every CTA streams pass 1 of its slice of wave s,
+// then pass 2 of its slice of wave s - lag (ecokv_params.sched_lag, 0 = 1).
+// Waves of a few heads make a key's second read an L2 hit; one wave (the
+// default) runs all of pass 1 first, which measured fastest so far: the
+// per-tile cost of the pipeline, not DRAM, bounds the small-wave schedules.
+static int tc_wave_units(const ecokv_params& p) {
   const long long U = (long long)p.n_layers * p.h_kv;
-  while (t > kTcMinTiles && U * ((p.n + 128LL * t - 1) / (128LL * t)) < kItemsWanted) t >>= 1;
-  return env_int("ECOKV_TC_TILES", t, kTcMinTiles, kTcMaxTiles);
+  const long long uw = p.sched_wave > 0 ? p.sched_wave : U;
+  return (int)(uw < U ? uw : U);
 }
-static int tc_chunk_keys(const ecokv_params& p) { return 128 * tc_tiles(p); }
+
+// Record slots per unit of the tensor-core passes (a bound over grids of up
+// to kTcMaxSms CTAs, so that it does not depend on the device).
+static int tc_records(const ecokv_params& p) {
+  const long long U = (long long)p.n_layers * p.h_kv;
+  const int T = (p.n + 127) / 128, uw = tc_wave_units(p);
+  const long long nw = (U + uw - 1) / uw, last = U - (nw - 1) * uw;
+  return tc_record_slots(T, (int)((uw < last ? uw : last) * T));
+}
 
 // SMs of the current device (cached per device).
 static int num_sms() {
@@ -110,13 +116,6 @@ static int num_sms() {
     cached[dev].store(n);
   }
   return cached[dev].load();
-}
-
-static int env_int(const char* name, int dflt, int lo, int hi) {
-  const char* v = getenv(name);
-  if (v == nullptr || *v == 0) return dflt;
-  const int x = atoi(v);
-  return x < lo ? lo : (x > hi ? hi : x);
 }
 
 // Keys forming the centroid of Eq. 1: all N, or with the non-window centroid
@@ -156,7 +155,7 @@ static FinalArgs final_args(const ecokv_params& p, const Layout& L, char* ws) {
   f.N = p.n;
   f.W = p.window;
   f.Tv = L.Tv;
-  f.nchunks = L.nchunks * L.p2slots;
+  f.nchunks = L.nchunks;
   f.budget = p.budget;
   f.pool = p.pool_kernel;
   f.ustat_stride = L.ustat_stride;
@@ -194,11 +193,15 @@ static CompactArgs compact_args(const ecokv_params& p, const void* K, const void
   return c;
 }
 
+// Device-side wait limit of a call: ecokv_params.timeout_us, 0 = 2 s.
+static unsigned long long wait_limit_ns(const ecokv_params& p) {
+  return (p.timeout_us ? (unsigned long long)p.timeout_us : 2000000ull) * 1000ull;
+}
+
 // Both streaming passes on the tensor cores in one launch (after clearing
 // the per-call counters).
 static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
-  const int tiles = tc_tiles(p);
-  const Layout L = make_layout(p, 128 * tiles, kTcP2Parts);
+  const Layout L = make_layout(p, tc_records(p));
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   TcArgs a{};
   a.U = L.U;
@@ -213,32 +216,21 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.Tv = L.Tv;
   a.kbar_n = kbar_count(p, L);
   a.q_rows = p.n_layers * p.h_q * p.window;
-  a.tiles_per_chunk = tiles;
-  a.nchunks = L.nchunks;
-  // pass 2 of unit u is scheduled lag units after its pass 1.  By default all
-  // of pass 1 runs first: pass-2 items then never wait for unit statistics,
-  // and the keys of a unit are gone from L2 by its pass 2 at any lag longer
-  // than the items in flight, so nothing is lost (ECOKV_LAG_P2 for tuning)
-  a.lag_p2 = env_int("ECOKV_LAG_P2", 1 << 20, 1, 1 << 20);
-  if (a.lag_p2 > L.U) a.lag_p2 = L.U;
-  // the pass-2 items of the last schedule steps are split in parts, so that
-  // the persistent CTAs run out of work at nearly the same time (the work
-  // after the last ticket is a part, not a whole item); only the steps that
-  // hold pass-2 items alone (the last lag_p2) are eligible
-  const int tail_items = a.lag_p2 * a.nchunks;
-  int nsplit = env_int("ECOKV_TAIL_SPLIT", num_sms(), 0, 1 << 30);
-  if (nsplit > tail_items) nsplit = tail_items;
-  a.nparts = env_int("ECOKV_TAIL_PARTS", kTcP2Parts, 1, kTcP2Parts);
-  if (tiles < a.nparts) a.nparts = tiles;
-  a.split_from = 2 * L.U * a.nchunks - nsplit;
-  a.total_tickets = a.split_from + a.nparts * nsplit;
+  a.T = (p.n + 127) / 128;
+  a.uw = tc_wave_units(p);
+  a.nw = (L.U + a.uw - 1) / a.uw;
+  a.lag = p.sched_lag > 0 ? p.sched_lag : 1;
+  if (a.lag > a.nw) a.lag = a.nw;
+  const int sms = num_sms();
+  a.P = sms < kTcMaxSms ? sms : kTcMaxSms;
+  a.rmax = L.nchunks;
   a.p1_stride = L.p1_stride;
   a.ustat_stride = L.ustat_stride;
+  a.stall_unit = (p.flags & ECOKV_FLAG_TEST_STALL) ? 0 : -1;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)p.d));
-  a.timeout_cycles = 4000000000LL;  // about 2 s of SM clock per wait
+  a.timeout_ns = wait_limit_ns(p);
   a.Q = Q;
   a.K = K;
-  a.norm2 = reinterpret_cast<float*>(ws + L.norm2);
   a.p1part = reinterpret_cast<float*>(ws + L.p1part);
   a.ustat = reinterpret_cast<float*>(ws + L.ustat);
   a.p2part = reinterpret_cast<float*>(ws + L.p2part);
@@ -247,14 +239,15 @@ static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const vo
   a.cosv = reinterpret_cast<float*>(ws + L.cosv);
   a.sync = reinterpret_cast<unsigned*>(ws + L.sync);
   a.status = reinterpret_cast<unsigned*>(ws + L.status);
-  if (launch_tc(K, a, s) != cudaSuccess) return ECOKV_ERR_CUDA;
+  if (launch_tc(K, a, s) != cudaSuccess) return ECOKV_ERR_CUDA;  // a grid of a.P CTAs
   return ECOKV_OK;
 }
 
 // CUDA-core streaming passes: fill the per-token arrays and unit statistics.
 static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const void* K, const void* Q, char* ws,
                                     cudaStream_t s) {
-  const Layout L = make_layout(p, kChunk);
+  if (p.flags & ECOKV_FLAG_TEST_STALL) return ECOKV_ERR_UNSUPPORTED;  // the stall exists on the tensor-core path
+  const Layout L = make_layout(p, simt_records(p));
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   const ScoreArgs a = score_args(p, L, K, Q, ws);
   if (launch_score_simt(a, dt, L.U, s) != cudaSuccess) return ECOKV_ERR_CUDA;
@@ -346,12 +339,13 @@ ecokv_status ecokv_check_params(const ecokv_params* p) {
   if (!(p->eps > 0.f) || !isfinite(p->eps) || !isfinite(p->tau)) return ECOKV_ERR_INVALID_ARG;
   const uint32_t known =
       ECOKV_FLAG_SC_MIXKV_SIGN | ECOKV_FLAG_LAMBDA_OVERRIDE | ECOKV_FLAG_VNORM_IMP | ECOKV_FLAG_CENTROID_NONWIN |
-      ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5 | ECOKV_FLAG_MAD | ECOKV_FLAG_FORCE_SIMT;
+      ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5 | ECOKV_FLAG_MAD | ECOKV_FLAG_FORCE_SIMT | ECOKV_FLAG_TEST_STALL;
   if ((p->flags & ~known) != 0u) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_WINSOR_1) && (p->flags & ECOKV_FLAG_WINSOR_5)) return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_MAD) && (p->flags & (ECOKV_FLAG_WINSOR_1 | ECOKV_FLAG_WINSOR_5)))
     return ECOKV_ERR_INVALID_ARG;
   if ((p->flags & ECOKV_FLAG_LAMBDA_OVERRIDE) && !isfinite(p->lambda_override)) return ECOKV_ERR_INVALID_ARG;
+  if (p->sched_wave < 0 || p->sched_lag < 0) return ECOKV_ERR_INVALID_ARG;
   if (p->d != kD) return ECOKV_ERR_UNSUPPORTED;
   if (p->n > kMaxN) return ECOKV_ERR_UNSUPPORTED;
   if ((long long)(p->h_q / p->h_kv) * p->window > kMaxRows) return ECOKV_ERR_UNSUPPORTED;
@@ -378,7 +372,7 @@ ecokv_status ecokv_score(const ecokv_params* p, ecokv_dtype dtype, const void* K
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
+  const Layout L = make_layout(*p, tc ? tc_records(*p) : simt_records(*p));
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.lambda = lambda;
@@ -402,7 +396,7 @@ ecokv_status ecokv_select(const ecokv_params* p, const float* S, int32_t* idx, v
   if (st != ECOKV_OK) return st;
   if (!idx || !aligned16(idx)) return ECOKV_ERR_INVALID_ARG;
   if (p->budget < p->n && p->n > p->window && (!S || !aligned16(S))) return ECOKV_ERR_INVALID_ARG;
-  const Layout L = make_layout(*p, kChunk);
+  const Layout L = make_layout(*p, simt_records(*p));
   FinalArgs f = final_args(*p, L, nullptr);
   f.S = const_cast<float*>(S);
   f.idx = idx;
@@ -423,7 +417,7 @@ ecokv_status ecokv_compact(const ecokv_params* p, ecokv_dtype dtype, const void*
   if (!aligned16(K) || !aligned16(V) || !aligned16(K_out) || !aligned16(V_out) || ((uintptr_t)idx & 3u))
     return ECOKV_ERR_INVALID_ARG;
   if (ws != nullptr && (!aligned16(ws) || ws_bytes < 256)) return ECOKV_ERR_WORKSPACE;
-  const Layout L = make_layout(*p, kChunk);
+  const Layout L = make_layout(*p, simt_records(*p));
   unsigned* status = ws ? reinterpret_cast<unsigned*>(static_cast<char*>(ws) + L.status) : nullptr;
   const CompactArgs c = compact_args(*p, K, V, idx, K_out, V_out, status);
   if (launch_compact(c, dtype, L.U, static_cast<cudaStream_t>(stream)) != cudaSuccess) return ECOKV_ERR_CUDA;
@@ -444,7 +438,7 @@ ecokv_status ecokv_evict_adaptive(const ecokv_params* p, ecokv_dtype dtype, cons
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
+  const Layout L = make_layout(*p, tc ? tc_records(*p) : simt_records(*p));
   const int n_keep = p->budget < p->n ? p->budget : p->n;
   const bool keep_all = p->budget >= p->n;
   // 1. every head's scores, into the workspace
@@ -506,7 +500,7 @@ static ecokv_status evict_impl(const ecokv_params* p, ecokv_dtype dtype, const v
   char* w = static_cast<char*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool tc = use_tensor_path(*p, dtype);
-  const Layout L = make_layout(*p, tc ? tc_chunk_keys(*p) : kChunk, tc ? kTcP2Parts : 1);
+  const Layout L = make_layout(*p, tc ? tc_records(*p) : simt_records(*p));
   FinalArgs f = final_args(*p, L, w);
   f.S = S;
   f.S_scratch = reinterpret_cast<float*>(w + L.sbuf);

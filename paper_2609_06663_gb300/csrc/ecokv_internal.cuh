@@ -36,16 +36,15 @@ struct DevStatus {
   unsigned detail;   // unit or item that raised it
 };
 
-// Byte offsets of the workspace regions for one parameter block and one
-// streaming chunk size (kChunk keys on the CUDA-core path, kTcChunk on the
-// tensor-core path).
+// Byte offsets of the workspace regions for one parameter block and a number
+// of partial-record slots per unit (chunks of kChunk keys on the CUDA-core
+// path, the slices a unit meets on the tensor-core path).
 struct Layout {
   int U;             // units = n_layers * h_kv
   int R;             // window rows per unit = (h_q / h_kv) * window
   int N, W, Tv;      // tokens, window, candidates
-  int chunk;         // keys per streaming chunk
-  int nchunks;       // ceil(N / chunk)
-  int p2slots;       // pass-2 partial slots per chunk (a chunk's pass-2 item may be split in parts)
+  int nchunks;       // record slots per unit: streaming chunks (CUDA-core passes) or slices met
+                     // (tensor-core passes)
   int p1_stride;     // floats per (unit, chunk) pass-1 partial: 2R + 2D
   int ustat_stride;  // floats per unit statistics record
   size_t status, sync, p1part, ustat, p2part, simp, dE, cosv, sbuf, norm2;
@@ -57,7 +56,7 @@ struct Layout {
   size_t sync_bytes; // bytes of the per-call counters cleared before each call
 };
 
-Layout make_layout(const ecokv_params& p, int chunk, int p2slots = 1);
+Layout make_layout(const ecokv_params& p, int nrec);
 
 // unit statistics record (floats):  [0,D) kbar | [D,2D) mu | [2D] ||kbar||^2 |
 //                                    [2D+1] ||mu||^2 | [2D+2, 2D+2+R) log2-LSE of the window rows

@@ -6,7 +6,9 @@
 // the host link); ecokv_evict then runs on those copies with V, K_out, V_out
 // and lambda left in host memory, so that the gather reads only the kept V
 // rows over the link and writes the outputs there directly; the indices,
-// made in the workspace, are copied back last.
+// made in the workspace, are copied back last.  With value-norm importance
+// (ECOKV_FLAG_VNORM_IMP) the norm kernel reads every row of V where it lies,
+// so then all of V crosses the link as well.
 //
 // Workspace layout: [ecokv_workspace_size bytes | K copy | Qwin copy | idx],
 // each region 256-byte aligned.

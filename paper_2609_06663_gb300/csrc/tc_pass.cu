@@ -1,47 +1,57 @@
-// Persistent tensor-core kernel for bf16 inputs: the whole eviction pass in
-// one launch on sm_103a.
+// Persistent tensor-core kernel for bf16 inputs: both streaming passes of the
+// eviction pass in one launch on sm_103a.
 //
-// Work is a global, ticket-ordered list of items:
-//   P1(u, c)  pass 1 over chunk c (up to 32 tiles of 128 keys) of unit u
-//             (u = (layer, KV head)): window logits (tcgen05 MMA, keys as M,
+// Work items (u = unit = (layer, KV head); a chunk is up to 64 tiles of 128
+// consecutive keys of one unit):
+//   P1(u, c)  pass 1 over chunk c: window logits (tcgen05 MMA, keys as M,
 //             window rows as N), per-row online-softmax partials, key norms,
 //             and the chunk sums of k and k/||k|| (a second tcgen05 MMA with the
 //             key tile as an MN-major operand against [1, w_hi, w_mid, w_lo]
-//             weight rows, w = 1/||k|| split into three bf16 terms).  The last P1 item of a unit folds the partials into the unit
-//             statistics (kbar, mu, per-row log2-sum-exp).
+//             weight rows, w = 1/||k|| split into three bf16 terms).
 //   P2(u, c)  pass 2: logits again plus five extra MMA columns holding k . kbar
 //             (kbar split into three bf16 terms) and k . mu (two terms), giving
 //             the importance vote, the cosine khat . mu, and d_E (Eq. 1) by the
-//             expansion of Sec. 4 from ||k||^2 (stored by pass 1).  Where that
-//             expansion cancels (d_E^2 below 2^-6 of ||k||^2 + ||kbar||^2, keys
-//             close to their centroid) the key is recomputed directly from its
-//             row in global memory.
-// Work is a global, ticket-ordered list of items.  Within a schedule step s
-// the list holds P1(s, *) then P2(s - lag_p2, *): pass 2 of a unit runs lag_p2
-// units after its pass 1 (a short lag re-reads the keys from L2, a long one
-// never waits for unit statistics; the host picks), and every item depends
-// only on items with smaller tickets: dispatch is deadlock-free without
-// co-residency.  Pass 2 leaves per-candidate arrays and per-chunk partial
-// sums; finalisation, selection and the gather of the kept rows run in the
-// next launches (finalize_select.cu).
+//             expansion of Sec. 4 from ||k||^2 (recomputed from the tile in
+//             shared memory).  Where that expansion cancels (d_E^2 below 2^-6
+//             of ||k||^2 + ||kbar||^2, keys close to their centroid) the key is
+//             recomputed directly from its row in global memory.
 //
-// Warp roles (512 threads, one CTA per SM): warp 0 takes tickets, resolves
-// dependencies (bounded spins on gpu-scope flags), loads the window queries
-// (TMA) and the unit statistics (bulk copy) and issues TMA loads of 32 KB key
-// tiles into a 5-stage ring; warp 1 issues the logits MMAs into up to four
-// TMEM accumulators; warp 3 issues the sum MMAs of pass-1 tiles (two more
-// accumulators) as soon as a tile's logits are done and its weights written,
-// and frees the stage; warp 2 counts finished pass-1 items and folds completed
-// units; warps 12-15 (key warps, one key per thread) compute the key norms
-// and the sum weights of each pass-1 tile as soon as it lands, store the norms
-// for pass 2, read the chunk sums, and hand the norms to the epilogue in pass
-// 2; warps 4-11 are the epilogue (one key per TMEM lane, window rows split in
-// two halves).  A stage is held only as long as its own tile needs it: the
-// number of key bytes in flight per SM, not the arithmetic, sets the pace.
-// setmaxnreg gives the two epilogue warpgroups 176 registers a thread and the
-// others 80.  Every mbarrier wait and spin is bounded: on timeout the kernel
-// records ECOKV_ERR_TIMEOUT, raises a gpu-wide abort flag, drains its own
-// copies and MMAs, frees TMEM and exits.
+// Schedule.  The chunks of all units, in unit order, form blocks of `blk`
+// chunks.  Tickets, taken from a global counter, run through steps: step s
+// holds the P1 items of block s, then the P2 items of block s - lag.  Pass 2
+// of a chunk therefore follows its pass 1 by about lag blocks of DRAM reads,
+// which the host keeps well inside L2: the second read of every key hits L2,
+// so K crosses the HBM interface once.  Every item depends only on items with
+// smaller tickets, so dispatch is deadlock-free without co-residency.  The
+// last P2 items may be split in parts (each with its own partial slot), so
+// that the CTAs run out of work together.
+//
+// Unit statistics (kbar, mu, ||kbar||^2, ||mu||^2, per-row log2-sum-exp): the
+// first CTA to start a P2 item of unit u claims the unit (an atomic on a
+// per-unit word); its epilogue warps wait until every P1 item of u has
+// arrived (a per-unit counter the stats warp of each CTA increments with
+// release semantics), fold the chunk partials in a fixed order with all 256
+// threads, publish the record and raise the unit's ready flag.  Other P2
+// items of u wait for that flag and read the record.  Nothing but the MMA and
+// the epilogue of a P2 item waits for it: the producer keeps loading key
+// tiles meanwhile.
+//
+// Warp roles (512 threads, one CTA per SM): warp 0 takes tickets and issues
+// TMA loads of the window queries and of 32 KB key tiles into a 5-stage ring;
+// warp 1 issues the logits MMAs into up to four TMEM accumulators; warp 3
+// issues the sum MMAs of pass-1 tiles (two more accumulators) as soon as a
+// tile's logits are done and its weights written, and frees the stage; warp 2
+// counts finished pass-1 items per unit; warps 12-15 (key warps, one key per
+// thread) compute the key norms of every tile as it lands (the sum weights in
+// pass 1, a hand-off to the epilogue in pass 2) and read the chunk sums;
+// warps 4-11 are the epilogue (one key per TMEM lane, window rows split in two
+// halves), which also folds or reads the unit statistics and writes the
+// statistics rows of the MMA operand at the start of a P2 item.  setmaxnreg
+// gives the two epilogue warpgroups 176 registers a thread and the others 80.
+// Every mbarrier wait and spin is bounded (a limit in nanoseconds of the
+// global timer): on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
+// gpu-wide abort flag, drains its own copies (key tiles and window queries)
+// and MMAs, frees TMEM and exits.
 
 #include <cuda.h>
 
@@ -58,6 +68,7 @@ namespace {
 using namespace ptx;
 
 constexpr int kIQ = 2;
+constexpr int kPrefetchTiles = 8;  // pass-1 tiles of an item prefetched into L2 when the item starts
 constexpr int kTile = 128;
 constexpr int kThreads = 512;
 constexpr int kEpi = 256;
@@ -74,14 +85,14 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSigmaCol = 256;
 constexpr uint32_t kEpiBar = 1;
 
-enum : int { kP1 = 0, kP2 = 1, kExit = 3 };
+enum : int { kP1 = 0, kP2 = 1, kFold = 2, kExit = 3 };
 
 constexpr int kNB = 4;                // pass-2 norm hand-off slots
 constexpr int kUstatMax = 2 * kD + 4 + kNPMax;  // floats of a unit statistics record (lse padded to NP rows)
 
 struct __align__(16) ItemDesc {
-  int type, u, chunk, part, i0, ntiles;
-  int pad[2];
+  int type, u, rec, i0, ntiles;  // rec: the item's record slot (its slice's index among the unit's slices)
+  int pad[3];
   float ust[kUstatMax];  // pass 2: copy of the unit statistics record (kbar, mu, norms, log2-LSE)
 };
 
@@ -107,8 +118,10 @@ struct __align__(1024) Smem {
   float nbuf[kNB][kTile];                        // pass-2 squared key norms, key warps -> epilogue
   uint64_t nfull[kNB], nempty[kNB];
   uint64_t xfull[kNB], xempty[kNB];             // first row half -> second row half, per pass-2 tile
-  uint64_t kpub[kIQ];    // key warps have published this item's key norms (gpu scope)
-  uint64_t p1done[kIQ];  // the epilogue has written this pass-1 item's partials
+  uint64_t kpub[kIQ];    // key warps have written this pass-1 item's chunk sums
+  uint64_t sready[kIQ];  // pass 2: unit statistics in desc.ust and statistics rows in qbuf (stats warp ->
+                         // MMA and epilogue)
+  float fold[512];       // epilogue scratch: combining the fold's thread groups
   uint32_t tmem_base;
   int epi_abort;         // an epilogue warp gave up a wait (read after a named barrier)
 };
@@ -119,6 +132,14 @@ static_assert(sizeof(Smem<8>) + 1024 <= 232448 && sizeof(Smem<16>) + 1024 <= 232
 static_assert(sizeof(ItemDesc) % 16 == 0 && offsetof(ItemDesc, ust) % 16 == 0, "bulk-copy target alignment");
 
 __device__ __forceinline__ unsigned* abort_flag(const TcArgs& a) { return a.sync + 1; }
+__device__ __forceinline__ unsigned* arrivals(const TcArgs& a, int u) { return a.sync + 4 + u; }
+__device__ __forceinline__ unsigned* stats_ready(const TcArgs& a, int u) { return a.sync + 4 + a.U + u; }
+
+__device__ __forceinline__ unsigned long long now_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
 
 __device__ void raise_abort(const TcArgs& a, unsigned code, unsigned detail) {
   if (atomicCAS(a.status, 0u, code) == 0u) a.status[1] = detail;
@@ -132,12 +153,12 @@ __device__ __forceinline__ bool aborted(const TcArgs& a) {
 // Bounded wait on an mbarrier phase; false on timeout or abort.
 __device__ bool wait_bar(uint64_t* bar, uint32_t parity, const TcArgs& a, unsigned where) {
   if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
+  const unsigned long long t0 = now_ns();
   for (unsigned spins = 1;; ++spins) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((spins & 63u) == 0u) {
       if (aborted(a)) return false;
-      if (clock64() - t0 > a.timeout_cycles) {
+      if (now_ns() - t0 > a.timeout_ns) {
         raise_abort(a, ECOKV_ERR_TIMEOUT, where);
         return false;
       }
@@ -145,81 +166,43 @@ __device__ bool wait_bar(uint64_t* bar, uint32_t parity, const TcArgs& a, unsign
   }
 }
 
-// Tiles of a chunk, and of part p (1..nparts) of it (its first tile in *t0);
-// part 0 is the whole chunk.
-__device__ __forceinline__ int chunk_tiles(const TcArgs& a, int chunk) {
-  return min(a.tiles_per_chunk, (a.N - chunk * a.tiles_per_chunk * kTile + kTile - 1) / kTile);
-}
-__device__ __forceinline__ int part_tiles(const TcArgs& a, int chunk, int part, int* t0) {
-  const int nt = chunk_tiles(a, chunk);
-  if (part == 0) {
-    if (t0) *t0 = 0;
-    return nt;
+// Wait for an mbarrier phase without regard to the abort flag, bounded: the
+// drain of copies in flight before a CTA leaves.
+__device__ void drain_bar(uint64_t* bar, uint32_t parity, const TcArgs& a) {
+  const unsigned long long t0 = now_ns();
+  while (!mbar_try_wait(bar, parity) && now_ns() - t0 < a.timeout_ns) {
   }
-  const int per = (nt + a.nparts - 1) / a.nparts, first = (part - 1) * per;
-  if (t0) *t0 = first;
-  return min(per, nt - first);
 }
 
-struct Item {
-  int type, u, chunk, part;
-  bool valid;
-};
-
-// Item of a ticket.  Schedule step s holds the P1 items of unit s and then
-// the P2 items of unit s - lag_p2; steps are numbered so that no ticket falls
-// outside [0, U): the first lag_p2 steps hold P1 items only, the last lag_p2
-// steps P2 items only, 2 * U * nchunks tickets in all.  lag_p2 = U runs all of
-// pass 1 before any of pass 2.
-__device__ Item decode(int ticket, const TcArgs& a) {
-  Item it{kExit, 0, 0, 0, true};
-  if (ticket >= a.total_tickets) return it;
-  int part = 0;
-  if (ticket >= a.split_from) {
-    // the last pass-2 items, each split in nparts consecutive parts
-    const int rel = ticket - a.split_from;
-    part = 1 + rel % a.nparts;
-    ticket = a.split_from + rel / a.nparts;
-  }
-  it.part = part;
-  const int nc = a.nchunks, L = a.lag_p2;
-  const int head = L * nc, body = (a.U - L) * 2 * nc;
-  if (ticket < head) {
-    it.type = kP1;
-    it.u = ticket / nc;
-    it.chunk = ticket - it.u * nc;
-  } else if (ticket < head + body) {
-    const int rel = ticket - head, st = rel / (2 * nc), slot = rel - st * 2 * nc;
-    if (slot < nc) {
-      it.type = kP1;
-      it.u = L + st;
-      it.chunk = slot;
-    } else {
-      it.type = kP2;
-      it.u = st;
-      it.chunk = slot - nc;
-    }
-  } else {
-    const int rel = ticket - head - body, v = rel / nc;
-    it.type = kP2;
-    it.u = a.U - L + v;
-    it.chunk = rel - v * nc;
-  }
-  it.valid = it.u >= 0 && it.u < a.U;
-  if (part > 0 && part_tiles(a, it.chunk, part, nullptr) <= 0) it.valid = false;  // a part past the chunk's end
-  return it;
+// Static schedule.  Wave w holds units [w uw, (w + 1) uw) (fewer in the last
+// wave), L = their tiles in unit order; it is cut into n = min(P, L)
+// contiguous slices, slice c covering wave tiles [floor(c L / n),
+// floor((c + 1) L / n)).  CTA c takes slice c of every wave.
+__device__ __forceinline__ int wave_tiles(const TcArgs& a, int w) { return min(a.uw, a.U - w * a.uw) * a.T; }
+__device__ __forceinline__ int slice_start(int c, int L, int n) { return (int)((long long)c * L / n); }
+// The slice holding wave tile o: the largest c with slice_start(c) <= o.
+__device__ __forceinline__ int slice_at(int o, int L, int n) {
+  return (int)(((long long)(o + 1) * n + L - 1) / L) - 1;
+}
+// The slices unit u meets: the first one, and how many (= its pass-1 records).
+__device__ __forceinline__ void unit_slices(const TcArgs& a, int u, int& c0, int& nrec) {
+  const int w = u / a.uw, L = wave_tiles(a, w), n = min(a.P, L);
+  const int o = (u - w * a.uw) * a.T;
+  c0 = slice_at(o, L, n);
+  nrec = slice_at(o + a.T - 1, L, n) - c0 + 1;
 }
 
-// Bounded spin on a gpu-scope flag written by another CTA.
-__device__ bool wait_flag(const unsigned* f, const TcArgs& a, unsigned where) {
-  const long long t0 = clock64();
-  while (ld_acquire(f) == 0u) {
+// Bounded spin until a gpu-scope counter written by other CTAs reaches
+// `target` (acquire); false on timeout or abort.
+__device__ bool wait_count(const unsigned* f, unsigned target, const TcArgs& a, unsigned where) {
+  const unsigned long long t0 = now_ns();
+  while (ld_acquire(f) < target) {
     if (aborted(a)) return false;
-    if (clock64() - t0 > a.timeout_cycles) {
+    if (now_ns() - t0 > a.timeout_ns) {
       raise_abort(a, ECOKV_ERR_TIMEOUT, where);
       return false;
     }
-    __nanosleep(128);
+    __nanosleep(64);
   }
   return true;
 }
@@ -237,93 +220,24 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // hold kbar split into three bf16 terms (hi, mid, lo), rows NP-5, NP-4 hold
 // mu_hi and mu_lo, all from the unit statistics copy (the last eight columns
 // of the accumulator belong to the second row half); the window queries in
-// rows 0..R-1 arrive by TMA.  Run by the 32 lanes of warp 0.
-__device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, float* ust, int lane) {
-  // rows past the window rows (padding and the statistics rows) get an
-  // infinite log-sum-exp, so that their vote terms are exactly zero
-  for (int r = a.R + lane; r < a.NP; r += 32) ust[ustat_lse() + r] = INFINITY;
-  for (int e = lane; e < 5 * 16; e += 32) {
-    const int which = e >> 4, j = e & 15;
-    const float* src = ust + (which < 3 ? ustat_kbar() : ustat_mu()) + j * 8;
-    const int term = which < 3 ? which : which - 3;  // 0 = hi, 1 = mid / lo, 2 = lo
-    float o[8];
+// rows 0..R-1 arrive by TMA.  Task e (0 <= e < 80) writes one 16-byte
+// vector: term row e / 16, dimensions 8 (e % 16) .. 8 (e % 16) + 7.
+__device__ void build_stat_rows(uint8_t* qb, const TcArgs& a, const float* ust, int e) {
+  const int which = e >> 4, j = e & 15;
+  const float* src = ust + (which < 3 ? ustat_kbar() : ustat_mu()) + j * 8;
+  const int term = which < 3 ? which : which - 3;  // 0 = hi, 1 = mid / lo, 2 = lo
+  float o[8];
 #pragma unroll
-    for (int t = 0; t < 8; ++t) {
-      const float x = src[t];
-      const float hi = __bfloat162float(__float2bfloat16_rn(x));
-      const float r1 = x - hi;
-      const float mid = __bfloat162float(__float2bfloat16_rn(r1));
-      o[t] = term == 0 ? hi : (which < 3 ? (term == 1 ? mid : r1 - mid) : r1);
-    }
-    const uint4 val = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
-                                 pack_bf16x2(o[6], o[7]));
-    *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(a.NP - 8 + which, j & 7)) = val;
+  for (int t = 0; t < 8; ++t) {
+    const float x = src[t];
+    const float hi = __bfloat162float(__float2bfloat16_rn(x));
+    const float r1 = x - hi;
+    const float mid = __bfloat162float(__float2bfloat16_rn(r1));
+    o[t] = term == 0 ? hi : (which < 3 ? (term == 1 ? mid : r1 - mid) : r1);
   }
-}
-
-// Fold every chunk's pass-1 partials of unit u into its statistics record,
-// one warp: lane l sums key dimensions 4l..4l+3 (16-byte loads) and combines
-// the (max, sum) pairs of window rows l, l + 32, ... online.  Loads go out in
-// batches so that the L2 latency is paid a few times per unit.  Chunk record:
-// [sum k (d)] [sum k/||k|| (d)] [row max (R4)] [row sum (R4)].
-__device__ void unit_reduce_warp(const TcArgs& a, int u, int lane) {
-  const int nch = a.nchunks;
-  const float* base = a.p1part + (size_t)u * nch * a.p1_stride;
-  float* us = a.ustat + (size_t)u * a.ustat_stride;
-  constexpr int kB = 8;
-  float4 sk = make_float4(0.f, 0.f, 0.f, 0.f), sh = sk;
-  for (int c0 = 0; c0 < nch; c0 += kB) {
-    float4 kv[kB], hv[kB];
-#pragma unroll
-    for (int j = 0; j < kB; ++j) {
-      const float4* p = reinterpret_cast<const float4*>(base + (size_t)min(c0 + j, nch - 1) * a.p1_stride);
-      kv[j] = __ldcg(p + lane);
-      hv[j] = __ldcg(p + kD / 4 + lane);
-    }
-#pragma unroll
-    for (int j = 0; j < kB; ++j)
-      if (c0 + j < nch) {
-        sk.x += kv[j].x; sk.y += kv[j].y; sk.z += kv[j].z; sk.w += kv[j].w;
-        sh.x += hv[j].x; sh.y += hv[j].y; sh.z += hv[j].z; sh.w += hv[j].w;
-      }
-  }
-  const float inv_n = 1.f / (float)a.N, inv_k = 1.f / (float)a.kbar_n;
-  const float4 kb = make_float4(sk.x * inv_k, sk.y * inv_k, sk.z * inv_k, sk.w * inv_k);
-  const float4 mu = make_float4(sh.x * inv_n, sh.y * inv_n, sh.z * inv_n, sh.w * inv_n);
-  reinterpret_cast<float4*>(us + ustat_kbar())[lane] = kb;
-  reinterpret_cast<float4*>(us + ustat_mu())[lane] = mu;
-  float ksq = (kb.x * kb.x + kb.y * kb.y) + (kb.z * kb.z + kb.w * kb.w);
-  float msq = (mu.x * mu.x + mu.y * mu.y) + (mu.z * mu.z + mu.w * mu.w);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    ksq += __shfl_xor_sync(0xffffffffu, ksq, o);
-    msq += __shfl_xor_sync(0xffffffffu, msq, o);
-  }
-  if (lane == 0) {
-    us[ustat_ksq()] = ksq;
-    us[ustat_musq()] = msq;
-  }
-  for (int r = lane; r < a.R; r += 32) {
-    float M = -INFINITY, Z = 0.f;
-    constexpr int kR = 16;
-    for (int c0 = 0; c0 < nch; c0 += kR) {
-      float mv[kR], zv[kR];
-#pragma unroll
-      for (int j = 0; j < kR; ++j) {
-        const float* p = base + (size_t)min(c0 + j, nch - 1) * a.p1_stride + 2 * kD;
-        mv[j] = __ldcg(p + r);
-        zv[j] = c0 + j < nch ? __ldcg(p + a.R4 + r) : 0.f;
-      }
-#pragma unroll
-      for (int j = 0; j < kR; ++j)
-        if (zv[j] > 0.f) {
-          const float Mn = fmaxf(M, mv[j]);
-          Z = Z * ex2(M - Mn) + zv[j] * ex2(mv[j] - Mn);
-          M = Mn;
-        }
-    }
-    us[ustat_lse() + r] = M + log2f(Z);
-  }
+  const uint4 val = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                               pack_bf16x2(o[6], o[7]));
+  *reinterpret_cast<uint4*>(qb + (j >> 3) * (a.NP * 128) + sw128(a.NP - 8 + which, j & 7)) = val;
 }
 
 // Joint (max, sum) of partial softmax sums: (m1, z1) + (m2, z2) with z
@@ -335,11 +249,88 @@ __device__ __forceinline__ void combine_maxsum(float& m, float& z, float m2, flo
   m = M;
 }
 
-// Reduce-scatter of RH (max, sum) rows over the 32 lanes of a warp: each
-// step exchanges half of the remaining rows with the partner lane, so lane l
-// ends with row (l >> shift) * per + j in m[j], z[j] (shift = 0, 1, 2 for
-// RH = 32 (or more), 16, 8; per = RH / 32 rows when RH > 32); lanes that share
-// a row hold the same value.
+// Fold the nch pass-1 records of unit u into its statistics record, by the
+// 256 epilogue threads (tid), with all loads of a thread issued together
+// (one round trip for up to 48 records).  Record: [sum k (d)] [sum k/||k||
+// (d)] [row max (R4)] [row sum (R4)].  Sums: thread (q, c) = (tid >> 7, tid &
+// 127) adds floats 2c, 2c + 1 of the records q, q + 2, ... in order; the two
+// groups are added in order.  Rows: thread (g, r) = (tid / R, tid % R), g <
+// G = min(8, 256 / R), combines the (max, sum) pairs of row r in the records
+// g, g + G, ... in order, then the G groups in order.  The record goes to the
+// unit's place in global memory.  Uses s_fold (512 floats) and named barrier
+// kEpiBar among the 256 threads.
+__device__ void fold_unit_stats(const TcArgs& a, int u, int nch, int tid, float* s_fold) {
+  const float* base = a.p1part + (size_t)u * a.rmax * a.p1_stride;
+  float* gus = a.ustat + (size_t)u * a.ustat_stride;
+  const int q = tid >> 7, c = tid & 127;
+  const int R = a.R, G = min(8, kEpi / R);
+  const bool lrow = tid < G * R;
+  const int g = lrow ? tid / R : 0, r = lrow ? tid - g * R : 0;
+  float sx = 0.f, sy = 0.f, M = -INFINITY, Z = 0.f;
+  constexpr int kS = 24, kL = 12;
+  for (int b = 0;; ++b) {
+    const int r0 = q + 2 * kS * b, l0 = g + G * kL * b;
+    if (r0 >= nch && (!lrow || l0 >= nch)) break;
+    float2 v[kS];
+    float mv[kL], zv[kL];
+#pragma unroll
+    for (int j = 0; j < kS; ++j)
+      v[j] = __ldcg(reinterpret_cast<const float2*>(base + (size_t)min(r0 + 2 * j, nch - 1) * a.p1_stride) + c);
+#pragma unroll
+    for (int j = 0; j < kL; ++j) {
+      const float* p = base + (size_t)min(l0 + G * j, nch - 1) * a.p1_stride + 2 * kD;
+      mv[j] = __ldcg(p + r);
+      zv[j] = __ldcg(p + a.R4 + r);
+    }
+#pragma unroll
+    for (int j = 0; j < kS; ++j)
+      if (r0 + 2 * j < nch) {
+        sx += v[j].x;
+        sy += v[j].y;
+      }
+#pragma unroll
+    for (int j = 0; j < kL; ++j)
+      if (lrow && l0 + G * j < nch && zv[j] > 0.f) combine_maxsum(M, Z, mv[j], zv[j]);
+  }
+  if (q == 1) {
+    s_fold[2 * c] = sx;
+    s_fold[2 * c + 1] = sy;
+  }
+  named_bar_sync(kEpiBar, kEpi);
+  if (q == 0) {
+    sx += s_fold[2 * c];
+    sy += s_fold[2 * c + 1];
+    // columns 2c, 2c + 1: sum of k for c < 64, sum of k/||k|| for c >= 64
+    const float sc = c < 64 ? 1.f / (float)a.kbar_n : 1.f / (float)a.N;
+    const float x = sx * sc, y = sy * sc;
+    __stcg(reinterpret_cast<float2*>(gus) + c, make_float2(x, y));
+    // ||kbar||^2 (warps 0, 1 of the group) and ||mu||^2 (warps 2, 3)
+    float sq = fmaf(x, x, y * y);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    if ((c & 31) == 0) s_fold[256 + (c >> 5)] = sq;
+  }
+  named_bar_sync(kEpiBar, kEpi);
+  if (tid == 0) {
+    gus[ustat_ksq()] = s_fold[256] + s_fold[257];
+    gus[ustat_musq()] = s_fold[258] + s_fold[259];
+  }
+  named_bar_sync(kEpiBar, kEpi);
+  if (lrow) {
+    s_fold[2 * tid] = M;
+    s_fold[2 * tid + 1] = Z;
+  }
+  named_bar_sync(kEpiBar, kEpi);
+  if (tid < R) {
+    float Mx = -INFINITY, Zx = 0.f;
+    for (int gg = 0; gg < G; ++gg) {
+      const float m2 = s_fold[2 * (gg * R + tid)], z2 = s_fold[2 * (gg * R + tid) + 1];
+      if (z2 > 0.f) combine_maxsum(Mx, Zx, m2, z2);
+    }
+    gus[ustat_lse() + tid] = Mx + log2f(Zx);
+  }
+}
+
 template <int RH>
 __device__ __forceinline__ void warp_reduce_scatter_maxsum(float (&m)[RH], float (&z)[RH], int lane) {
   int n = RH;
@@ -386,8 +377,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < kIQ; ++i) {
       mbar_init(&s.item_full[i], 1);
       mbar_init(&s.item_empty[i], 1 + 8 + kKeyWarps + 2);  // MMA commit + epilogue + key warps + stats + sum warps
-      mbar_init(&s.p1done[i], 8);
       mbar_init(&s.qfull[i], 1);
+      mbar_init(&s.sready[i], 1);
     }
     for (int i = 0; i < 4; ++i) {
       mbar_init(&s.tmem_full[i], 1);
@@ -446,6 +437,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
     const uint32_t bmask = (1u << nbuf_log) - 1u;
     uint32_t tcount = 0, pcount = 0;
+    uint32_t spar = 0u;  // per slot: parity of the next sready phase (completed by P2 items only)
     auto epi_sync = [&]() -> bool {
       if (!ok) s.epi_abort = 1;
       named_bar_sync(kEpiBar, kEpi);
@@ -462,9 +454,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       const ItemDesc& d = s.desc[slot];
       const int type = d.type;
       if (type == kExit) break;
-      const int u = d.u, chunk = d.chunk, i0 = d.i0, ntiles = d.ntiles;
+      const int u = d.u, rec = d.rec, i0 = d.i0, ntiles = d.ntiles;
 
-      if (type == kP1) {
+      if (type == kFold) {
+        // unit statistics: once every P1 item of unit u has arrived, fold
+        // their partials with all 256 threads and publish the record
+        int c0, nrec;
+        unit_slices(a, u, c0, nrec);
+        const unsigned need = (unsigned)nrec + (u == a.stall_unit ? 1u : 0u);
+        if (tid == 0) ok = wait_count(arrivals(a, u), need, a, 30u);
+        if (!epi_sync()) {
+          ok = false;
+          break;
+        }
+        fold_unit_stats(a, u, nrec, tid, s.fold);
+        named_bar_sync(kEpiBar, kEpi);
+        if (tid == 0) {
+          __threadfence();
+          st_release(stats_ready(a, u), 1u);
+        }
+      } else if (type == kP1) {
         float m[RH], z[RH];
 #pragma unroll
         for (int c = 0; c < RH; ++c) {
@@ -555,7 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        float* part = a.p1part + ((size_t)u * a.nchunks + chunk) * a.p1_stride;
+        float* part = a.p1part + ((size_t)u * a.rmax + rec) * a.p1_stride;
         if (tid < a.R) {
           const int hh = tid / RH, c = tid % RH;
           float Mx = -INFINITY;
@@ -570,11 +579,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           part[2 * kD + tid] = Mx;
           part[2 * kD + a.R4 + tid] = Z;
         }
-        // the stats warp counts the item once all eight warps have written
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s.p1done[slot]);
+        // once the key warps' chunk sums are written too, one gpu-scope
+        // release publishes the item (every partial write is ordered before
+        // it by the barrier and the kpub wait)
+        named_bar_sync(kEpiBar, kEpi);
+        if (tid == 0) {
+          ok = wait_bar(&s.kpub[slot], qphase, a, 19u);
+          if (ok) red_add_release(arrivals(a, u), 1u);
+          else s.epi_abort = 1;
+        }
       } else {  // kP2
-        ok = __all_sync(0xffffffffu, wait_bar(&s.qfull[slot], qphase, a, 18u));  // statistics copy landed
+        // the stats warp has copied the unit statistics and built the
+        // statistics rows
+        ok = __all_sync(0xffffffffu, wait_bar(&s.sready[slot], (spar >> slot) & 1u, a, 18u));
+        spar ^= 1u << slot;
         const float* lse = d.ust + ustat_lse();
         const float* kbv = d.ust + ustat_kbar();
         const float ksq = d.ust[ustat_ksq()];
@@ -688,15 +706,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float x = s.red6[w4][tid];
             acc = tid == 1 ? fminf(acc, x) : tid == 2 ? fmaxf(acc, x) : acc + x;
           }
-          // the chunk's slot of this part; the first part also fills every
-          // slot no part writes with the identity of its reduction
-          float* p = a.p2part + ((size_t)u * a.nchunks + chunk) * kTcP2Parts * kP2Stride;
-          const int part = d.part;
-          p[(part > 0 ? part - 1 : 0) * kP2Stride + tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
-          if (part <= 1) {
+          // the item's record slot; the unit's first record also fills every
+          // slot past the unit's records with the identity of its reduction
+          float* p = a.p2part + (size_t)u * a.rmax * kP2Stride;
+          p[rec * kP2Stride + tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
+          if (rec == 0) {
+            int c0, nrec;
+            unit_slices(a, u, c0, nrec);
             const float idn = tid == P2_MIN_DE ? INFINITY : tid == P2_MAX_DE ? -INFINITY : 0.f;
-            for (int q = 1; q < kTcP2Parts; ++q)
-              if (part == 0 || q >= a.nparts || part_tiles(a, chunk, q + 1, nullptr) <= 0) p[q * kP2Stride + tid] = idn;
+            for (int q = nrec; q < a.rmax; ++q) p[q * kP2Stride + tid] = idn;
           }
         }
       }
@@ -709,104 +727,124 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ scheduler + TMA producer
     int stage = 0;
     uint32_t sphase = 0;
-    uint32_t used_bits = 0u, par_bits = 0u;  // per stage: loaded at least once / parity of loads
-    const uint64_t pol_keep = l2_policy_evict_last(), pol_drop = l2_policy_evict_first();
-    for (int seq = 0; ok;) {
-      int ticket = 0;
-      if (lane == 0) ticket = (int)atomicAdd(a.sync, 1u);
-      ticket = __shfl_sync(0xffffffffu, ticket, 0);
-      const Item it = decode(ticket, a);
-      if (!it.valid) continue;
+    uint32_t used_bits = 0u, par_bits = 0u;    // per key stage: loaded at least once / parity of loads
+    uint32_t qused_bits = 0u, qpar_bits = 0u;  // the same per window-query slot
+    // the first read of a key is kept in L2 for its second read when pass 2
+    // follows pass 1 by a few blocks; the second read is the last
+    const uint64_t pol_p1 = a.lag < a.nw ? l2_policy_evict_last() : l2_policy_evict_first();
+    const uint64_t pol_p2 = l2_policy_evict_first();
+    int seq = 0;
+    // One item: publish its descriptor (and start its window-query copy),
+    // then load its key tiles into the ring.
+    auto emit = [&](int type, int u, int t_lo, int ntiles, int rec) -> bool {
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
-      if (lane == 0) {
-        ok = wait_bar(&s.item_empty[slot], qphase ^ 1u, a, 1u);
-        if (ok && it.type == kP2) {
-          ok = wait_flag(a.sync + 4 + a.U + it.u, a, 2u);
-          fence_proxy_async_global();  // the statistics are read next by a bulk copy (async proxy)
-        }
+      const int i0 = t_lo * kTile;
+      const uint64_t pol = type == kP1 ? pol_p1 : pol_p2;
+      if (type == kP1) {
+        // the item's first pass-1 tiles go to L2 now, ahead of the
+        // shared-memory ring (a few only: more floods the memory queues)
+        for (int e = lane; e < 2 * min(ntiles, kPrefetchTiles); e += 32)
+          tma_prefetch_3d(&tmK, (e & 1) * 64, i0 + (e >> 1) * kTile, u, pol_p1);
       }
-      ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
-      if (!ok) break;
+      bool good = true;
+      if (lane == 0) good = wait_bar(&s.item_empty[slot], qphase ^ 1u, a, 1u);
+      if (__shfl_sync(0xffffffffu, good, 0) == 0) return false;
       ItemDesc& d = s.desc[slot];
-      int t0 = 0;
-      const int ntiles = it.type == kExit ? 0 : part_tiles(a, it.chunk, it.part, &t0);
-      const int i0 = (it.chunk * a.tiles_per_chunk + t0) * kTile;
       if (lane == 0) {
-        d.type = it.type;
-        d.u = it.u;
-        d.chunk = it.chunk;
-        d.part = it.part;
+        d.type = type;
+        d.u = u;
+        d.rec = rec;
         d.i0 = i0;
         d.ntiles = ntiles;
-      }
-      if (it.type == kP1 || it.type == kP2) {
-        // window queries by TMA (swizzled in flight); pass 2 also copies the
-        // unit statistics record
-        const uint32_t ust_bytes = (uint32_t)a.ustat_stride * 4u;
-        if (lane == 0) {
-          const int layer = it.u / a.h_kv, head = it.u % a.h_kv;
+        if (type == kP1 || type == kP2) {
+          // window queries by TMA (swizzled in flight); the MMA (pass 1) or
+          // the stats warp (pass 2) waits for them, not this warp
+          const int layer = u / a.h_kv, head = u % a.h_kv;
           const int qrow = (layer * a.h_q + head * a.g) * a.W;
-          mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u + (it.type == kP2 ? ust_bytes : 0u));
+          mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u);
           tma_load_2d(s.qbuf[slot], &tmQ, &s.qfull[slot], 0, qrow);
           tma_load_2d(s.qbuf[slot] + a.NP * 128, &tmQ, &s.qfull[slot], 64, qrow);
-          if (it.type == kP2) bulk_load(d.ust, a.ustat + (size_t)it.u * a.ustat_stride, ust_bytes, &s.qfull[slot]);
-          ok = wait_bar(&s.qfull[slot], qphase, a, 16u);
+          qused_bits |= 1u << slot;
+          qpar_bits ^= 1u << slot;
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
-        if (!ok) break;
-        if (it.type == kP2) build_stat_rows(s.qbuf[slot], a, d.ust, lane);
       }
-      fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.item_full[slot]);
       ++seq;
-      if (it.type == kExit) {
-        // no work left for this CTA: the next launch (finalisation) may be
-        // scheduled on SMs as they drain; it waits for this grid's completion
-        // before reading anything
-        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-        break;
-      }
-      for (int t = 0; t < ntiles && ok; ++t) {
+      for (int t = 0; t < ntiles; ++t) {
         if (lane == 0) {
-          ok = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
-          if (ok) {
+          good = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
+          if (good) {
             mbar_expect_tx(&s.full[stage], kTileBytes);
             const int y = i0 + t * kTile;
-            // with pass 2 close behind pass 1 (a short lag), pass 1 keeps its
-            // keys in L2 for it; with all of pass 1 first no key survives in L2
-            // until its pass 2, and keeping them only crowds out the data the
-            // finalisation reads next, so every load is evict-first
-            const uint64_t pol = (it.type == kP1 && a.lag_p2 < a.U) ? pol_keep : pol_drop;
-            tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, it.u, pol);
-            tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, it.u, pol);
+            tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, u, pol);
+            tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, u, pol);
             used_bits |= 1u << stage;
             par_bits ^= 1u << stage;
           }
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        if (__shfl_sync(0xffffffffu, good, 0) == 0) return false;
         if (++stage == kStages) {
           stage = 0;
           sphase ^= 1u;
         }
       }
+      return true;
+    };
+    // Step s: pass 1 of this CTA's slice of wave s; the folds of the units of
+    // wave s - 1 it owns (unit u belongs to CTA u mod P, so that no CTA folds
+    // in every wave); pass 2 of its slice of wave s - lag.  A fold holds its
+    // CTA's epilogue until the unit's last pass-1 item has arrived; a step
+    // later every CTA has long finished wave s - 1, and pass 2 of those units
+    // (lag >= 2) comes a step later still.
+    const int c = blockIdx.x;
+    for (int st = 0; st < a.nw + a.lag && ok; ++st) {
+      for (int ph = 0; ph < 3 && ok; ++ph) {  // 0: pass 1, 1: folds, 2: pass 2
+        const int w = ph == 0 ? st : (ph == 1 ? st - 1 : st - a.lag);
+        if (w < 0 || w >= a.nw) continue;
+        if (ph == 1) {
+          const int u1 = min((w + 1) * a.uw, a.U);
+          for (int u = w * a.uw + ((c - w * a.uw) % a.P + a.P) % a.P; u < u1 && ok; u += a.P)
+            ok = emit(kFold, u, 0, 0, 0);
+          continue;
+        }
+        const int L = wave_tiles(a, w), n = min(a.P, L);
+        if (c >= n) continue;
+        const int g0 = w * a.uw * a.T;  // the wave's first tile, counted over all units
+        const int lo = g0 + slice_start(c, L, n), hi = g0 + slice_start(c + 1, L, n);
+        for (int u = lo / a.T; u * a.T < hi && ok; ++u) {
+          const int t_lo = max(lo, u * a.T) - u * a.T, t_hi = min(hi, (u + 1) * a.T) - u * a.T;
+          int c0, nrec;
+          unit_slices(a, u, c0, nrec);
+          ok = emit(ph == 0 ? kP1 : kP2, u, t_lo, t_hi - t_lo, c - c0);
+        }
+      }
+    }
+    if (ok) {
+      // no work left for this CTA: the next launch (finalisation) may be
+      // scheduled on SMs as they drain; it waits for this grid's completion
+      // before reading anything
+      ok = emit(kExit, 0, 0, 0, 0);
+      asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     }
     if (!ok && lane == 0) {
-      // let this CTA's copies in flight land before its shared memory goes away
+      // let this CTA's copies in flight land before its shared memory goes
+      // away: the last key tile of every stage and the last window-query copy
+      // of every slot (a slot or stage is reloaded only after its previous
+      // copy was consumed, so only the last one can be pending)
       for (int st = 0; st < kStages; ++st)
-        if (used_bits & (1u << st)) {
-          const uint32_t last = ((par_bits >> st) & 1u) ^ 1u;  // parity of the last load's phase
-          const long long t0 = clock64();
-          while (!mbar_try_wait(&s.full[st], last) && clock64() - t0 < a.timeout_cycles) {
-          }
-        }
+        if (used_bits & (1u << st)) drain_bar(&s.full[st], ((par_bits >> st) & 1u) ^ 1u, a);
+      for (int sl = 0; sl < kIQ; ++sl)
+        if (qused_bits & (1u << sl)) drain_bar(&s.qfull[sl], ((qpar_bits >> sl) & 1u) ^ 1u, a);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
       int stage = 0;
       uint32_t sphase = 0, tcount = 0;
+      uint32_t spar = 0u;  // per slot: parity of the next sready phase (completed by P2 items only)
+      uint32_t qpar = 0u;  // per slot: parity of the next qfull phase (completed by P1 and P2 items)
       const uint32_t idesc_l = idesc_bf16(128, a.NP, false, false);
       for (int seq = 0; ok; ++seq) {
         const int slot = seq % kIQ;
@@ -815,7 +853,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         const ItemDesc& d = s.desc[slot];
         const int type = d.type, ntiles = d.ntiles;
         if (type == kExit) break;
-        if (!(ok = wait_bar(&s.qfull[slot], qphase, a, 17u))) break;  // queries landed (already observed by warp 0)
+        if (type == kP1 || type == kP2) qpar ^= 1u << slot;
+        if (type == kP1) {
+          // the window queries landed
+          if (!(ok = wait_bar(&s.qfull[slot], ((qpar >> slot) & 1u) ^ 1u, a, 17u))) break;
+        } else if (type == kP2) {
+          // the stats warp has the unit statistics and wrote the statistics rows
+          if (!(ok = wait_bar(&s.sready[slot], (spar >> slot) & 1u, a, 17u))) break;
+          spar ^= 1u << slot;
+        }
         tc_fence_after();
         const uint32_t qb = smem_u32(s.qbuf[slot]);
         for (int t = 0; t < ntiles; ++t) {
@@ -844,9 +890,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) {
         mma_commit(&s.drain);
-        const long long t0 = clock64();
-        while (!mbar_try_wait(&s.drain, 0u) && clock64() - t0 < a.timeout_cycles) {
-        }
+        drain_bar(&s.drain, 0u, a);
       }
     }
   } else if (warp == 3) {
@@ -898,18 +942,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) {
         mma_commit(&s.drain2);
-        const long long t0 = clock64();
-        while (!mbar_try_wait(&s.drain2, 0u) && clock64() - t0 < a.timeout_cycles) {
-        }
+        drain_bar(&s.drain2, 0u, a);
       }
     }
   } else if (warp == 2) {
     // ------------------------------------------------ stats warp
-    // Counts finished pass-1 items per unit (gpu-scope atomic); the item that
-    // completes a unit folds its chunk partials into the unit statistics and
-    // releases pass 2 of the unit.  Runs beside the epilogue so that neither
-    // the count's round trip nor the fold holds up the tiles.
-    uint32_t p1par = 0u;  // per slot: parity of the next p1done phase
+    // Readies the unit statistics of every P2 item, about one item ahead of
+    // the epilogue: waits for the unit's ready flag (raised by the fold
+    // item), copies the record into the item descriptor, gives the rows past
+    // R an infinite log-sum-exp (their vote terms are then exactly zero) and,
+    // once the window queries have landed, writes the statistics rows of the
+    // MMA operand over them.
+    uint32_t qpar = 0u;  // per slot: parity of the next qfull phase (completed by P1 and P2 items)
     for (int seq = 0; ok; ++seq) {
       const int slot = seq % kIQ;
       const uint32_t qphase = (uint32_t)(seq / kIQ) & 1u;
@@ -917,26 +961,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       const ItemDesc& d = s.desc[slot];
       const int type = d.type, u = d.u;
       if (type == kExit) break;
-      if (type == kP1) {
-        // the epilogue's partials and the key warps' norms of the item are written
-        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.p1done[slot], (p1par >> slot) & 1u, a, 27u)))) break;
-        p1par ^= 1u << slot;
-        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.kpub[slot], qphase, a, 19u)))) break;
+      if (type == kP1 || type == kP2) qpar ^= 1u << slot;
+      if (type == kP2) {
+        float* ust = s.desc[slot].ust;
+        if (lane == 0) ok = wait_count(stats_ready(a, u), 1u, a, 31u);
+        ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        if (!ok) break;
+        __syncwarp();  // lane 0's acquire orders the record's loads below
+        const float4* g = reinterpret_cast<const float4*>(a.ustat + (size_t)u * a.ustat_stride);
+        for (int e4 = lane; e4 < a.ustat_stride / 4; e4 += 32) reinterpret_cast<float4*>(ust)[e4] = __ldcg(g + e4);
+        __syncwarp();
+        for (int r = a.R + lane; r < a.NP; r += 32) ust[ustat_lse() + r] = INFINITY;
+        if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.qfull[slot], ((qpar >> slot) & 1u) ^ 1u, a, 27u)))) break;
+        for (int e = lane; e < 5 * 16; e += 32) build_stat_rows(s.qbuf[slot], a, ust, e);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.sready[slot]);
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s.item_empty[slot]);  // free the slot before the long part
-      if (type == kP1) {
-        // the arrival is a gpu-scope release of everything this CTA wrote for
-        // the item (the mbarrier waits above ordered it before this thread)
-        unsigned old = 0u;
-        if (lane == 0) old = atom_add_acq_rel(a.sync + 4 + u, 1u);
-        old = __shfl_sync(0xffffffffu, old, 0);
-        if (old == (unsigned)(a.nchunks - 1)) {
-          unit_reduce_warp(a, u, lane);
-          __syncwarp();
-          if (lane == 0) st_release(a.sync + 4 + a.U + u, 1u);
-        }
-      }
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
     }
   } else if (warp >= kKeyWarp0) {
     // ------------------------------------------------ key warps (12..15)
@@ -954,26 +997,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.full[stage], sphase, a, 22u)))) break;
         const int i = i0 + t * kTile + kk;
         const bool valid = i < a.N;
-        if (type == kP1) {
-          // squared norm of this thread's key (packed fp32 pairs), kept for
-          // pass 2, and the sum weights w = 1/||k|| in three bf16 terms
-          float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        // squared norm of this thread's key (packed fp32 pairs), the same
+        // arithmetic in both passes
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int hb = 0; hb < 2; ++hb) {
-            const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
+        for (int hb = 0; hb < 2; ++hb) {
+          const uint8_t* row = s.ktile[stage] + hb * (kTileBytes / 2) + kk * 128;
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
-              sq_acc_bf16x2(v.x, acc[0], acc[1]);
-              sq_acc_bf16x2(v.y, acc[2], acc[3]);
-              sq_acc_bf16x2(v.z, acc[4], acc[5]);
-              sq_acc_bf16x2(v.w, acc[6], acc[7]);
-            }
+          for (int c = 0; c < 8; ++c) {
+            const uint4 v = *reinterpret_cast<const uint4*>(row + ((c ^ (kk & 7)) << 4));
+            sq_acc_bf16x2(v.x, acc[0], acc[1]);
+            sq_acc_bf16x2(v.y, acc[2], acc[3]);
+            sq_acc_bf16x2(v.z, acc[4], acc[5]);
+            sq_acc_bf16x2(v.w, acc[6], acc[7]);
           }
-          const float n2 = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
-          if (valid) __stcs(a.norm2 + (size_t)u * a.N + i, n2);  // read once, by pass 2
+        }
+        const float n2 = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.empty[stage]);  // done with the key tile
+        if (type == kP1) {
+          // the sum weights w = 1/||k|| in three bf16 terms
           const float w = valid ? rsqrtf(fmaxf(n2, 1e-24f)) : 0.f;
           const __nv_bfloat16 whi = __float2bfloat16_rn(w);
           const float r1 = w - __bfloat162float(whi);
@@ -990,15 +1033,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.wready[stage]);
         } else {
-          // pass 2: the keys are only needed by the MMA; the norms pass 1
-          // stored go to the epilogue through shared memory
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.empty[stage]);
+          // pass 2: the norm goes to the epilogue through shared memory
           const uint32_t nb = p2count % kNB, nph = (p2count / kNB) & 1u;
           ++p2count;
-          const float n2 = valid ? __ldcs(a.norm2 + (size_t)u * a.N + i) : 0.f;
           if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nempty[nb], nph ^ 1u, a, 23u)))) break;
-          s.nbuf[nb][kk] = n2;
+          s.nbuf[nb][kk] = valid ? n2 : 0.f;
           __syncwarp();
           if (lane == 0) mbar_arrive(&s.nfull[nb]);
         }
@@ -1020,7 +1059,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&s.sigma_empty[sb]);
-        float* part = a.p1part + ((size_t)u * a.nchunks + d.chunk) * a.p1_stride;
+        float* part = a.p1part + ((size_t)u * a.rmax + d.rec) * a.p1_stride;
         part[kk] = __uint_as_float(v[0]);
         part[kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
       }
@@ -1062,8 +1101,20 @@ cudaError_t launch_rh(const CUtensorMap& tm, const CUtensorMap& tq, const TcArgs
     if (e != cudaSuccess) return e;
     g_attr_set[dev][rh_i].store(true);
   }
-  tc_evict_kernel<RH><<<g_num_sms[dev].load(), kThreads, smem, st>>>(tm, tq, a);
-  return cudaGetLastError();
+  // a cooperative launch: every CTA of the grid is resident at once (the
+  // static schedule has CTAs wait for other CTAs' pass-1 items), or the
+  // launch fails
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)a.P);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tc_evict_kernel<RH>, tm, tq, a);
 }
 
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -1089,6 +1140,14 @@ EncodeTiledFn encode_fn() {
 }  // namespace
 
 size_t tc_smem_bytes() { return sizeof(Smem<32>) + 1024; }
+
+int tc_record_slots(int T, int Lmin) {
+  // slices of a wave of L >= Lmin tiles cut in n = min(P, L) pieces, P <=
+  // kTcMaxSms, hold at least s = max(1, floor(Lmin / kTcMaxSms)) tiles; a
+  // unit's T consecutive tiles meet at most ceil((T - 1) / s) + 1 of them
+  const int s = Lmin / kTcMaxSms > 1 ? Lmin / kTcMaxSms : 1;
+  return (T - 1 + s - 1) / s + 1;
+}
 
 int tc_rows_half(int R) {
   const int r4 = (R + 3) & ~3;

@@ -21,6 +21,7 @@ ECOKV_FLAG_WINSOR_1 = 0x10
 ECOKV_FLAG_WINSOR_5 = 0x20
 ECOKV_FLAG_MAD = 0x40
 ECOKV_FLAG_FORCE_SIMT = 0x100
+ECOKV_FLAG_TEST_STALL = 0x80000000
 ECOKV_NOALLOC_SCRATCH_BYTES = 16 << 20   # fixed scratch of ecokv_evict_noalloc, per device
 ECOKV_OK, ECOKV_ERR_INVALID_ARG, ECOKV_ERR_UNSUPPORTED, ECOKV_ERR_WORKSPACE = 0, 1, 2, 3
 ECOKV_ERR_CUDA, ECOKV_ERR_TIMEOUT, ECOKV_ERR_DEVICE_INDEX = 4, 5, 6
@@ -45,7 +46,8 @@ class ecokv_params(ctypes.Structure):
                 ("n", ctypes.c_int32), ("d", ctypes.c_int32), ("window", ctypes.c_int32),
                 ("budget", ctypes.c_int32), ("pool_kernel", ctypes.c_int32),
                 ("alpha", ctypes.c_float), ("beta", ctypes.c_float), ("tau", ctypes.c_float),
-                ("eps", ctypes.c_float), ("flags", ctypes.c_uint32), ("lambda_override", ctypes.c_float)]
+                ("eps", ctypes.c_float), ("flags", ctypes.c_uint32), ("lambda_override", ctypes.c_float),
+                ("sched_wave", ctypes.c_int32), ("sched_lag", ctypes.c_int32), ("timeout_us", ctypes.c_uint32)]
 
     def as_dict(self) -> dict:
         return {f: getattr(self, f) for f, _ in self._fields_}
@@ -210,11 +212,13 @@ def ecokv_device_status(ws, stream=None) -> int:
 
 # ---------------------------------------------------------------- torch helpers
 def make_params(*, n_layers, h_kv, h_q, n, d=128, window, budget, pool_kernel=5, alpha=0.8, beta=0.6,
-                tau=0.0, eps=1e-6, flags=0, lambda_override=0.0) -> ecokv_params:
+                tau=0.0, eps=1e-6, flags=0, lambda_override=0.0, sched_wave=0, sched_lag=0,
+                timeout_us=0) -> ecokv_params:
     p = ecokv_params()
     for k, v in dict(n_layers=n_layers, h_kv=h_kv, h_q=h_q, n=n, d=d, window=window, budget=budget,
                      pool_kernel=pool_kernel, alpha=alpha, beta=beta, tau=tau, eps=eps, flags=flags,
-                     lambda_override=lambda_override).items():
+                     lambda_override=lambda_override, sched_wave=sched_wave, sched_lag=sched_lag,
+                     timeout_us=timeout_us).items():
         setattr(p, k, v)
     return p
 

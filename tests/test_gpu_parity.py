@@ -89,6 +89,25 @@ def test_small_shapes(case, path):
     run_and_compare(small_workload(seed=11, **case), flags=E.ECOKV_FLAG_FORCE_SIMT if path == "simt" else 0)
 
 
+# Streaming schedules of the tensor-core kernel: waves of one head to all of
+# them, lags from one wave to all of pass 1 first.
+SCHEDULES = [(1, 1), (1, 3), (2, 1), (5, 1), (3, 2), (6, 1)]
+
+
+@pytest.mark.parametrize("wave,lag", SCHEDULES, ids=lambda v: str(v))
+def test_streaming_schedules(wave, lag):
+    w = small_workload(5000, h_kv=2, group=7, window=8, budget=500, pool_kernel=5, dtype="bf16", n_layers=3,
+                       clustered=True)
+    run_and_compare(w, sched_wave=wave, sched_lag=lag)
+
+
+def test_streaming_schedule_many_units():
+    """Sixty heads of 1000 keys (8 tiles): slices that span several heads and
+    heads split over several slices."""
+    w = small_workload(1000, h_kv=4, group=2, window=4, budget=100, pool_kernel=5, dtype="bf16", n_layers=15)
+    run_and_compare(w, units=[(0, 0), (3, 1), (7, 2), (14, 3)])
+
+
 @pytest.mark.parametrize("flags,extra", [
     (O.FLAG_SC_MIXKV_SIGN, dict(alpha=0.0, beta=0.0)),          # MixKV special case
     (O.FLAG_LAMBDA_OVERRIDE, dict(lambda_override=0.0)),         # SnapKV importance only

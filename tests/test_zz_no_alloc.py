@@ -1,6 +1,6 @@
 """ecokv_evict_noalloc (workspace held by the library, nothing allocated by the
-call) against ecokv_evict with a caller workspace, on two calls in a row, and
-its host-side size check.  The file name sorts last so that the entry point is
+call) against ecokv_evict with a caller workspace, bit for bit, on two calls in
+a row, and its host-side size check.  The file name sorts last so that the entry point is
 exercised both alone and after every other test in the same process."""
 import numpy as np
 import pytest
@@ -8,7 +8,7 @@ import torch
 
 from paper_2609_06663_gb300 import ecokv as E
 from paper_2609_06663_gb300.workloads import make_inputs, small_workload, workload
-from tests.parity import TOL, check_rows, check_selection, oracle_params, score_error
+from tests.parity import check_rows
 
 DEV = "cuda"
 
@@ -59,17 +59,17 @@ def test_noalloc_matches_workspace_entry_two_calls(pair):
         idx, Ko, Vo, S, lam, code = E.evict_noalloc(p, K, V, Q, want_scores=True)
         torch.cuda.synchronize()
         assert code == 0, E.ecokv_status_string(code)
-        tol = TOL[w.dtype]
-        op = oracle_params(p)
-        S_ref = S_r.cpu().double().numpy()
-        S_got = S.cpu().double().numpy()
+        # the same kernels on the same inputs with the same schedule: every
+        # output is bit for bit the one the caller-workspace entry returns
+        # (a stale or misplaced scratch region would show here)
+        what = w.name
+        assert torch.equal(S, S_r), f"{what}: scores differ from ecokv_evict"
+        assert torch.equal(lam, lam_r), f"{what}: lambda differs from ecokv_evict"
+        assert torch.equal(idx, idx_r), f"{what}: indices differ from ecokv_evict"
+        assert torch.equal(Ko, Ko_r) and torch.equal(Vo, Vo_r), f"{what}: gathered rows differ"
+        # and the pass itself is sound: rows are the ones idx names
         for h in range(w.h_kv):
             for l in range(w.n_layers):
-                what = f"{w.name} unit ({l},{h})"
-                assert score_error(S_got[l, h], S_ref[l, h]) <= tol, what
-                assert abs(float(lam[l, h]) - float(lam_r[l, h])) <= tol, what
-                ref = {"S": S_ref[l, h], "idx": idx_r[l, h].cpu().numpy()}
-                check_selection(idx[l, h].cpu().numpy(), ref, op, tol, what)
-                check_rows(K[l, h], idx[l, h], Ko[l, h], what)
-                check_rows(V[l, h], idx[l, h], Vo[l, h], what)
-        assert np.isfinite(S_got).all()
+                check_rows(K[l, h], idx[l, h], Ko[l, h], f"{what} unit ({l},{h})")
+                check_rows(V[l, h], idx[l, h], Vo[l, h], f"{what} unit ({l},{h})")
+        assert np.isfinite(S.cpu().numpy()).all()
