@@ -37,6 +37,8 @@ sys.path.insert(0, ROOT)
 METRIC = "KV tokens evicted/sec per layer at 1 GB300; % of HBM roofline (GB/s)"
 UNIT = "tokens/s"
 FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 126 << 20       # GB300 L2
+FLUSH_BYTES = 256 << 20    # written between timed steps when the inputs would fit in L2
 
 
 def parse_args():
@@ -59,6 +61,9 @@ def parse_args():
                          "mad: MAD scaling in place of the min-max of Eq. 2 (ECOKV_FLAG_MAD)")
     ap.add_argument("--cpu-sample-units", type=int, default=0, help="0 = auto (about 10-30 s of CPU work)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="the bandwidth sweep instead of one workload: one layer, 8 KV / 32 query heads, bf16, "
+                         "budget 10 %%, N = 2^10 .. 2^17, W in {1, 4, 16, 32}; one JSON line per point")
     return ap.parse_args()
 
 
@@ -294,6 +299,10 @@ def main():
     if args.impl == "reference":
         run_reference(args, w, rank, world, cores)
         return
+    if args.sweep:
+        if rank == 0:
+            run_sweep(args)
+        return
 
     import torch.distributed as dist
     if world > 1:
@@ -346,6 +355,10 @@ def main():
         step()
     torch.cuda.synchronize(dev)
     assert E.ecokv_device_status(ws, stream) == 0
+    # inputs that L2 could hold between steps are flushed out of it before
+    # every timed step (a 256 MB write outside the timed region)
+    in_bytes = (K.numel() + V.numel() + Q.numel()) * K.element_size()
+    flush_buf = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev) if in_bytes < 2 * L2_BYTES else None
 
     def barrier():
         if world > 1:
@@ -359,12 +372,23 @@ def main():
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     barrier()
-    ev0.record(stream)
-    for i in range(args.steps):
-        step()
-    ev1.record(stream)
-    barrier()
-    ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
+    if flush_buf is None:
+        ev0.record(stream)
+        for i in range(args.steps):
+            step()
+        ev1.record(stream)
+        barrier()
+        ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
+    else:
+        pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in range(args.steps)]
+        for a_, b_ in pairs:
+            flush_buf.zero_()
+            a_.record(stream)
+            step()
+            b_.record(stream)
+        barrier()
+        ms = max_over_ranks(sum(a_.elapsed_time(b_) for a_, b_ in pairs), world, dev)
     # per-kernel durations: K more steps with events recorded by the library
     # between its launches (streaming kernel | finalize/select | compaction)
     # on the same stream; the events order the launches strictly, so this
@@ -375,6 +399,8 @@ def main():
             e.record(stream)  # creates the event handle
     barrier()
     for i in range(args.steps):
+        if flush_buf is not None:
+            flush_buf.zero_()
         E.ecokv_set_stage_events(stage_ev[i])
         step()
     E.ecokv_set_stage_events(None)
@@ -466,10 +492,15 @@ def main():
 
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "value_definition": "cache rows processed per second: every (layer, KV head) row of the prefill is "
+                            "scored and either kept or evicted, L * H_kv * N per step; the rows evicted per "
+                            "second are config.evicted_rows_per_s",
         "warmup": max(3, args.warmup), "ms_per_step": round(ms_step, 5), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
         "data": "synthetic (seeded anisotropic + clustered/temporally correlated keys; no dataset)",
-        "config": {**w.describe(), "workload": w.name, "l2": "inputs larger than L2 (no flush)",
+        "config": {**w.describe(), "workload": w.name,
+                   "l2": "inputs larger than L2 (no flush)" if flush_buf is None else
+                   "L2 flushed before every timed step (256 MB write outside the timed region)",
                    "variant": {"adaptive": "layer-wide budget (ecokv_evict_adaptive)",
                                "vnorm": "value-norm importance (ECOKV_FLAG_VNORM_IMP)",
                                "pyramid": f"per-layer budgets, PyramidKV beta 20: {budgets}",
@@ -494,6 +525,84 @@ def main():
         dist.destroy_process_group()
 
 
+def run_sweep(args) -> None:
+    """The bandwidth sweep on GPU 0: one layer of 8 KV / 32 query heads, bf16,
+    budget 10 %, N = 2^10 .. 2^17, W in {1, 4, 16, 32}.  Per point: 3 warm-up
+    calls, then --steps timed calls of ecokv_evict, each after a 256 MB L2
+    flush (outside the timed region), CUDA events around each call (median),
+    and as many calls with the library's stage events for the per-kernel
+    times.  Prints one JSON line per point."""
+    import torch
+
+    from paper_2609_06663_gb300 import ecokv as E
+    from paper_2609_06663_gb300.workloads import make_inputs, sweep_workload
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    peak, peak_kind = measured_peaks()
+    flush_buf = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    steps = max(5, args.steps)
+    for n in [1 << k for k in range(10, 18)]:
+        for win in (1, 4, 16, 32):
+            w = sweep_workload(n, win)
+            K, V, Q = make_inputs(w, device=dev)
+            p = E.make_params(n_layers=w.n_layers, h_kv=w.h_kv, h_q=w.h_q, n=w.n, d=w.d, window=w.window,
+                              budget=w.budget, pool_kernel=w.pool_kernel)
+            ws = E.alloc_workspace(p, dev)
+            n_keep = min(p.budget, w.n)
+            idx = torch.empty(w.n_layers, w.h_kv, n_keep, dtype=torch.int32, device=dev)
+            Ko = torch.empty(w.n_layers, w.h_kv, n_keep, w.d, dtype=K.dtype, device=dev)
+            Vo = torch.empty_like(Ko)
+            dt = E.dtype_code(K)
+
+            def step():
+                code = E.ecokv_evict(p, dt, K, V, Q, idx, Ko, Vo, None, None, ws, ws.numel(), stream)
+                if code:
+                    raise E.EcokvError(code, "ecokv_evict")
+
+            for _ in range(3):
+                step()
+            torch.cuda.synchronize(dev)
+            assert E.ecokv_device_status(ws, stream) == 0
+            pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                     for _ in range(steps)]
+            for a_, b_ in pairs:
+                flush_buf.zero_()
+                a_.record(stream)
+                step()
+                b_.record(stream)
+            stage_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+            for evs in stage_ev:
+                for e in evs:
+                    e.record(stream)
+            for evs in stage_ev:
+                flush_buf.zero_()
+                E.ecokv_set_stage_events(evs)
+                step()
+            E.ecokv_set_stage_events(None)
+            torch.cuda.synchronize(dev)
+            ms = statistics.median(a_.elapsed_time(b_) for a_, b_ in pairs)
+            stage_ms = [statistics.median(evs[j].elapsed_time(evs[j + 1]) for evs in stage_ev) for j in range(3)]
+            bm = byte_model(w)
+            gbs = lambda b, t: b / (t * 1e-3) / 1e9
+            print(json.dumps({
+                "sweep": "bandwidth sweep (one layer, 8 KV / 32 query heads, bf16, budget 10 %)",
+                "workload": w.name, "n": n, "window": win, "budget": w.budget,
+                "path": "tensor-core streaming kernel" if launches_per_call(w) == 3 else "CUDA-core passes",
+                "ms_per_call": round(ms, 5), "tokens_per_s": round(w.units * n / (ms * 1e-3), 1),
+                "evicted_rows_per_s": round(w.units * max(0, n - w.budget) / (ms * 1e-3), 1),
+                "alg_gbs": round(gbs(bm["alg"], ms), 1), "bl_gbs": round(gbs(bm["bl"], ms), 1),
+                "alg_frac": round(gbs(bm["alg"], ms) / peak, 4), "bl_frac": round(gbs(bm["bl"], ms) / peak, 4),
+                "stages_ms": {"streaming": round(stage_ms[0], 5), "finalize_select": round(stage_ms[1], 5),
+                              "compact": round(stage_ms[2], 5)},
+                "streaming_frac": round(gbs(bm["k"] + bm["q"], stage_ms[0]) / peak, 4),
+                "peak_gbs": peak, "peak_kind": f"{peak_kind} copy bandwidth (hbm_gbs)",
+                "timing": f"median of {steps} calls, each after a 256 MB L2 flush"}), flush=True)
+            del K, V, Q, ws, idx, Ko, Vo
+            torch.cuda.empty_cache()
+
+
 def run_reference(args, w, rank: int, world: int, cores: int) -> None:
     """The oracle timed as it stands, on host cores; rank 0 only."""
     if rank != 0:
@@ -513,6 +622,9 @@ def run_reference(args, w, rank: int, world: int, cores: int) -> None:
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "f64", "data": "synthetic", "impl": "reference",
            "config": {**w.describe(), "workload": w.name}, "cpu_baseline": cpu,
+           "timing": {"ms_per_step": "projected from the sampled rate: one step's L * H_kv * N rows divided by "
+                                     f"the oracle's rows per second over {nu} sampled (layer, head) units per "
+                                     "timed repetition; the whole step is not run on the CPU"},
            "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
 

@@ -69,7 +69,7 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
 #define ECOKV_FLAG_VNORM_IMP       0x4u /* S_imp(i) = pooled vote(i) * ||v_i||_2 (Sec. 5.2 combines the value
                                             norm with the window attention; the form is a reading).  Needs V:
                                             the ecokv_evict* entry points; ecokv_score returns
-                                            ECOKV_ERR_UNSUPPORTED.  Heads of up to 32768 candidates
+                                            ECOKV_ERR_UNSUPPORTED.  Heads of up to 131072 candidates
                                             (n - window), else ECOKV_ERR_UNSUPPORTED. */
 #define ECOKV_FLAG_CENTROID_NONWIN 0x8u /* the centroid kbar of Eq. 1 over the n - window candidates only
                                             (Appendix B's alternative to Algorithm 1 step 5; all keys when
@@ -78,12 +78,12 @@ typedef enum { ECOKV_F32 = 0, ECOKV_BF16 = 1 } ecokv_dtype;
                                              floor(p (n - W - 1)) and ceil((1 - p)(n - W - 1)) (0-based, no
                                              interpolation), p = 1 % (Appendix B's normalisation ablation) */
 #define ECOKV_FLAG_WINSOR_5        0x20u /* the same with p = 5 %; at most one of the two.  Both: heads of up
-                                             to 32768 candidates, else ECOKV_ERR_UNSUPPORTED */
+                                             to 131072 candidates, else ECOKV_ERR_UNSUPPORTED */
 #define ECOKV_FLAG_MAD             0x40u /* MAD scaling in place of the min-max of Eq. 2 (the same ablation):
                                              s_E = logistic((d_E - med) / (MAD + eps)), med the median of d_E
                                              over the candidates and MAD the median of |d_E - med| (an even
                                              count's median is the mean of its two middle values).  Not with
-                                             a WINSOR flag (ECOKV_ERR_INVALID_ARG); heads of up to 32768
+                                             a WINSOR flag (ECOKV_ERR_INVALID_ARG); heads of up to 131072
                                              candidates, else ECOKV_ERR_UNSUPPORTED */
 #define ECOKV_FLAG_FORCE_SIMT      0x100u /* run the CUDA-core passes even where the tensor-core kernel applies */
 #define ECOKV_FLAG_TEST_STALL      0x80000000u /* fault injection for tests of the bounded waits: the statistics of

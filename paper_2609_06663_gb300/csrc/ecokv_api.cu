@@ -255,7 +255,8 @@ static ecokv_status run_simt_passes(const ecokv_params& p, ecokv_dtype dt, const
 }
 
 // Scores (and the top-k) of every unit: one cluster per unit when the unit
-// fits eight CTAs, one CTA per unit otherwise.
+// fits a cluster (up to sixteen CTAs of 8192 candidates), one CTA per unit
+// otherwise.
 // Value-norm importance: reject heads the cluster finalize does not take
 // (before anything is launched), else the norms' launch and their place.
 static ecokv_status vnorm_check(const ecokv_params& p, const Layout& L) {

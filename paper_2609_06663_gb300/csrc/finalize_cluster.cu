@@ -49,29 +49,34 @@ constexpr int kCThreads = 256;
 constexpr int kCWarps = kCThreads / 32;
 constexpr int kHalo = 16;  // pooling halo kept in shared memory (kernel <= 33)
 
-template <int kJ>
+// Shapes (kSh): 0 = 16 candidates a thread, up to 8 CTAs; 1 = 32 a thread,
+// up to 4 CTAs; 2 = 32 a thread, up to 16 CTAs (clusters past the portable 8,
+// for units of 32769 to 131072 candidates; their larger exchange buffers
+// would cost the 4-CTA shape occupancy).
+template <int kSh>
 struct Shape {
-  static constexpr int kCap = kCThreads * kJ;          // candidates a CTA owns
-  static constexpr int kMaxCluster = kJ == 16 ? 8 : 4;  // CTAs a unit may take
-  static constexpr int kQ = kCap + 2 * kHalo;          // staged raw votes
+  static constexpr int kJ = kSh == 0 ? 16 : 32;                            // candidates a thread owns
+  static constexpr int kCap = kCThreads * kJ;                              // candidates a CTA owns
+  static constexpr int kMaxCluster = kSh == 0 ? 8 : (kSh == 1 ? 4 : 16);  // CTAs a unit may take
+  static constexpr int kQ = kCap + 2 * kHalo;                              // staged raw votes
 };
 
 // Padded shared-memory index of staged position q.
 __device__ __forceinline__ int pad_idx(int q) { return q + (q >> 5); }
 
-template <int kJ>
+template <int kSh>
 struct ClusterSmem {
   // raw vote of candidate lo - kHalo + q at raw[pad_idx(q)]
-  float raw[Shape<kJ>::kQ + Shape<kJ>::kQ / 32 + 1];
+  float raw[Shape<kSh>::kQ + Shape<kSh>::kQ / 32 + 1];
   unsigned whist[kCWarps][256];  // per radix pass, each warp's own histogram
   // Written by the peers (distributed shared memory stores): per radix pass
   // the histogram of every rank (double-buffered across passes), the S_div
   // extrema and the counts above / equal to the threshold of every rank.
-  unsigned hall[2][Shape<kJ>::kMaxCluster][256];
-  float ext_all[Shape<kJ>::kMaxCluster][2];
-  double simp_all[Shape<kJ>::kMaxCluster];  // value-norm importance: every rank's sum of S_imp
-  double wsum_all[Shape<kJ>::kMaxCluster];  // winsorised min-max / MAD scaling: every rank's sum of s_E terms
-  int cnt_all[Shape<kJ>::kMaxCluster][2];
+  unsigned hall[2][Shape<kSh>::kMaxCluster][256];
+  float ext_all[Shape<kSh>::kMaxCluster][2];
+  double simp_all[Shape<kSh>::kMaxCluster];  // value-norm importance: every rank's sum of S_imp
+  double wsum_all[Shape<kSh>::kMaxCluster];  // winsorised min-max / MAD scaling: every rank's sum of s_E terms
+  int cnt_all[Shape<kSh>::kMaxCluster][2];
   float red[kCWarps][8];  // per-warp partials
   float edge[32];         // pooling edge values
   float sc[8];            // broadcast scalars
@@ -112,12 +117,12 @@ __device__ __forceinline__ void push_all(cg::cluster_group& cl, T* obj, T v, int
 // kVar: the value-norm importance, winsorised min-max and MAD scaling
 // variants are compiled in (their code is left out of the default kernel, whose register budget it
 // would cost).
-template <int kMode, int kJ, bool kVar>
+template <int kMode, int kSh, bool kVar>
 __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArgs f) {
   constexpr bool kSelect = kMode != 0;
-  constexpr int kCap = Shape<kJ>::kCap, kMaxC = Shape<kJ>::kMaxCluster;
+  constexpr int kJ = Shape<kSh>::kJ, kCap = Shape<kSh>::kCap, kMaxC = Shape<kSh>::kMaxCluster;
   extern __shared__ __align__(16) uint8_t fc_smem[];
-  ClusterSmem<kJ>& sm = *reinterpret_cast<ClusterSmem<kJ>*>(fc_smem);
+  ClusterSmem<kSh>& sm = *reinterpret_cast<ClusterSmem<kSh>*>(fc_smem);
   cg::cluster_group cl = cg::this_cluster();
   // The peers must have started before the first store into their shared
   // memory: this arrival is waited for just before it.
@@ -708,29 +713,29 @@ __global__ void __launch_bounds__(kCThreads, 4) finalize_cluster_kernel(FinalArg
   // CTAs may leave independently.
 }
 
-template <int kJ>
-cudaError_t set_smem_attrs() {
-  const int bytes = (int)sizeof(ClusterSmem<kJ>);
-  cudaError_t e;
-  if ((e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                bytes)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                bytes)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(finalize_cluster_kernel<0, kJ, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                bytes)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(finalize_cluster_kernel<1, kJ, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                bytes)) != cudaSuccess)
-    return e;
-  return cudaFuncSetAttribute(finalize_cluster_kernel<2, kJ, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              bytes);
+template <int kSh>
+cudaError_t set_attrs() {
+  const int bytes = (int)sizeof(ClusterSmem<kSh>);
+  const void* kernels[5] = {(const void*)finalize_cluster_kernel<0, kSh, false>,
+                            (const void*)finalize_cluster_kernel<1, kSh, false>,
+                            (const void*)finalize_cluster_kernel<0, kSh, true>,
+                            (const void*)finalize_cluster_kernel<1, kSh, true>,
+                            (const void*)finalize_cluster_kernel<2, kSh, false>};
+  for (const void* k : kernels) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && Shape<kSh>::kMaxCluster > 8)
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
-template <int kJ>
+template <int kSh>
 cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cudaStream_t s) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)(U * C), 1, 1);
   cfg.blockDim = dim3(kCThreads, 1, 1);
-  cfg.dynamicSmemBytes = sizeof(ClusterSmem<kJ>);
+  cfg.dynamicSmemBytes = sizeof(ClusterSmem<kSh>);
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -742,42 +747,89 @@ cudaError_t launch_shape(const FinalArgs& f, int U, int C, bool select_only, cud
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   const bool var = f.vnorm != nullptr || f.wlo != nullptr || f.mad != nullptr;
-  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kJ, false>, f);
+  if (select_only) return cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<2, kSh, false>, f);
   if (f.idx == nullptr)
-    return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ, true>, f)
-               : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kJ, false>, f);
-  return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ, true>, f)
-             : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kJ, false>, f);
+    return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kSh, true>, f)
+               : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<0, kSh, false>, f);
+  return var ? cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kSh, true>, f)
+             : cudaLaunchKernelEx(&cfg, finalize_cluster_kernel<1, kSh, false>, f);
+}
+
+// Per device: the attributes set, and whether clusters of 16 CTAs of the
+// long shape can be resident (cudaOccupancyMaxActiveClusters > 0).
+std::atomic<int> g_setup[64];  // 0 = not yet, 1 = set, clusters of 16 unavailable, 2 = set and available
+
+int device_setup() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
+  int st = g_setup[dev].load();
+  if (st != 0) return st;
+  if (set_attrs<0>() != cudaSuccess || set_attrs<1>() != cudaSuccess) return -1;
+  st = 1;
+  if (set_attrs<2>() == cudaSuccess) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(16u * 16u, 1, 1);
+    cfg.blockDim = dim3(kCThreads, 1, 1);
+    cfg.dynamicSmemBytes = sizeof(ClusterSmem<2>);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 16;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, (const void*)finalize_cluster_kernel<1, 2, false>, &cfg) == cudaSuccess &&
+        n > 0)
+      st = 2;
+  }
+  cudaGetLastError();  // an unavailable configuration leaves no error behind
+  g_setup[dev].store(st);
+  return st;
+}
+
+// Shape and cluster size for units of Tv candidates; shape -1 when no cluster
+// shape takes them.
+void pick_shape(int Tv, int long_ok, int& sh, int& C) {
+  const int t = Tv > 0 ? Tv : 1;
+  const int C16 = (t + Shape<0>::kCap - 1) / Shape<0>::kCap;
+  const int C32 = (t + Shape<1>::kCap - 1) / Shape<1>::kCap;
+  if (C16 <= 4) {
+    sh = 0;
+    C = C16;
+  } else if (C32 <= Shape<1>::kMaxCluster) {
+    sh = 1;
+    C = C32;
+  } else if (C32 <= (long_ok ? Shape<2>::kMaxCluster : 8)) {
+    sh = 2;
+    C = C32;
+  } else {
+    sh = -1;
+    C = 0;
+  }
 }
 
 }  // namespace
 
 bool cluster_finalize_fits(int Tv) {
-  const int t = Tv > 0 ? Tv : 1;
-  const int C16 = (t + Shape<16>::kCap - 1) / Shape<16>::kCap;
-  const int C32 = (t + Shape<32>::kCap - 1) / Shape<32>::kCap;
-  return C16 > 4 ? C32 <= Shape<32>::kMaxCluster : C16 <= Shape<16>::kMaxCluster;
+  const int st = device_setup();
+  if (st < 0) return false;
+  int sh, C;
+  pick_shape(Tv, st == 2, sh, C);
+  return sh >= 0;
 }
 
-// Scores (and with f.idx the top-k) of every unit, or with select_only the
-// top-k of the scores in f.S; one cluster per unit; cudaErrorNotSupported
-// when Tv exceeds what eight CTAs of 4096 (or four of 8192) candidates hold.
 cudaError_t launch_finalize_cluster(const FinalArgs& f, int U, bool select_only, cudaStream_t s) {
-  const int Tv = f.Tv > 0 ? f.Tv : 1;
-  const int C16 = (Tv + Shape<16>::kCap - 1) / Shape<16>::kCap;
-  const int C32 = (Tv + Shape<32>::kCap - 1) / Shape<32>::kCap;
-  const bool wide = C16 > 4;
-  if (wide ? C32 > Shape<32>::kMaxCluster : C16 > Shape<16>::kMaxCluster) return cudaErrorNotSupported;
-  static std::atomic<bool> attr_set[64];  // a racing thread repeats the idempotent setup
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!attr_set[dev].load()) {
-    if ((e = set_smem_attrs<16>()) != cudaSuccess || (e = set_smem_attrs<32>()) != cudaSuccess) return e;
-    attr_set[dev].store(true);
+  const int st = device_setup();
+  if (st < 0) return cudaErrorUnknown;
+  int sh, C;
+  pick_shape(f.Tv, st == 2, sh, C);
+  switch (sh) {
+    case 0: return launch_shape<0>(f, U, C, select_only, s);
+    case 1: return launch_shape<1>(f, U, C, select_only, s);
+    case 2: return launch_shape<2>(f, U, C, select_only, s);
   }
-  return wide ? launch_shape<32>(f, U, C32, select_only, s) : launch_shape<16>(f, U, C16, select_only, s);
+  return cudaErrorNotSupported;
 }
 
 }  // namespace ecokv

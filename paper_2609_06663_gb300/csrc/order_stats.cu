@@ -5,7 +5,9 @@
 // One CTA per unit: its Tv <= 32768 distances are read in coalesced order
 // into shared memory as order-preserving keys, 64 thread-contiguous keys per
 // thread (padded so that a quarter-warp's 16-byte reads fall in distinct
-// banks), and an MSB-first radix select on the keys finds two ranks at once:
+// banks), and an MSB-first radix select on the keys finds two ranks at once
+// (longer rows are read from L2 until the keys left under the ranks'
+// prefixes fit those slots, see os_select2_long):
 // - the row's smallest and largest keys give the prefix every key shares;
 // - one digit of up to 12 bits just below it, counted by direct atomics into
 //   a block-wide histogram (the keys spread over its bins), and a suffix
@@ -142,6 +144,8 @@ __device__ __forceinline__ void os_scan(OsSmem& sm, int shift, int w, int tid) {
   __syncthreads();
 }
 
+__device__ __forceinline__ void os_tail(unsigned* seg, int n, OsSmem& sm, int left, int tid);
+
 // The ka-th and kb-th largest of the staged keys, into sm.pfx[0] and
 // sm.pfx[1]; the thread's keys at seg (nv of them) are reordered.  Enters
 // after a barrier that ends the staging.
@@ -213,7 +217,12 @@ __device__ __forceinline__ void os_select2(unsigned* seg, int nv, OsSmem& sm, in
     for (int r = 0; r < 4; ++r)
       if (4 * c4 + r < nv && ((kk[r] & m0) == p0 || (kk[r] & m1) == p1)) seg[n++] = kk[r];
   }
-  // remaining digits over the short lists
+  os_tail(seg, n, sm, left, tid);
+}
+
+// The remaining digits (left bits below both prefixes) over the thread's
+// short list of n keys at seg, the keys under either prefix.
+__device__ __forceinline__ void os_tail(unsigned* seg, int n, OsSmem& sm, int left, int tid) {
   while (left > 0) {
     const int w = min(kOsDigit, left), shift = left - w;
     const unsigned dm = (1u << w) - 1u;
@@ -227,6 +236,83 @@ __device__ __forceinline__ void os_select2(unsigned* seg, int nv, OsSmem& sm, in
     os_scan(sm, shift, w, tid);
     left = shift;
   }
+}
+
+// The ka-th and kb-th largest keys of a row too long for the stage (T >
+// kOsThreads * kOsPer), into sm.pfx[0] and sm.pfx[1]: the row is read from
+// global memory (L2) for the shared prefix and then for whole radix digits,
+// until every thread's keys under either prefix (of its positions tid, tid +
+// kOsThreads, ...) fit its kOsPer stage slots; those keys are then copied to
+// the slots at seg and the remaining digits run over them as for a short row.
+template <bool kDev>
+__device__ void os_select2_long(const float* xr, int T, float m, unsigned* seg, OsSmem& sm, int ka, int kb, int tid) {
+  const int lane = tid & 31, warp = tid >> 5;
+  unsigned lo = 0xffffffffu, hi = 0u;
+  for (int q = tid; q < T; q += kOsThreads) {
+    const unsigned k = os_key<kDev>(__ldg(xr + q), m);
+    lo = min(lo, k);
+    hi = max(hi, k);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  if (lane == 0) {
+    sm.red[0][warp] = lo;
+    sm.red[1][warp] = hi;
+  }
+  __syncthreads();
+  lo = sm.red[0][0];
+  hi = sm.red[1][0];
+  for (int w = 1; w < kOsWarps; ++w) {
+    lo = min(lo, sm.red[0][w]);
+    hi = max(hi, sm.red[1][w]);
+  }
+  const int common = __clz(lo ^ hi);  // 32 when every key is equal
+  const unsigned cmask = common == 32 ? 0xffffffffu : ~(0xffffffffu >> common);
+  if (tid < 2) {
+    sm.pfx[tid] = lo & cmask;
+    sm.mask[tid] = cmask;
+    sm.rem[tid] = (unsigned)(tid == 0 ? ka : kb);
+  }
+  __syncthreads();  // the state is set (and sm.red read) before any thread goes on
+  int left = 32 - common;
+  while (left > 0) {
+    const unsigned p0 = sm.pfx[0], m0 = sm.mask[0], p1 = sm.pfx[1], m1 = sm.mask[1];
+    unsigned cnt = 0u;
+    for (int q = tid; q < T; q += kOsThreads) {
+      const unsigned k = os_key<kDev>(__ldg(xr + q), m);
+      cnt += ((k & m0) == p0 || (k & m1) == p1) ? 1u : 0u;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cnt = max(cnt, __shfl_xor_sync(0xffffffffu, cnt, o));
+    if (lane == 0) sm.red[0][warp] = cnt;
+    __syncthreads();
+    unsigned mx = 0u;
+    for (int w = 0; w < kOsWarps; ++w) mx = max(mx, sm.red[0][w]);
+    if (mx <= (unsigned)kOsPer) break;  // the same decision in every thread
+    // one digit over the whole row (os_scan's barriers order the next
+    // iteration's writes to sm.red after these reads)
+    const int w = min(kOsDigit, left), shift = left - w;
+    const unsigned dm = (1u << w) - 1u;
+    const bool same = p0 == p1 && m0 == m1;
+    for (int q = tid; q < T; q += kOsThreads) {
+      const unsigned k = os_key<kDev>(__ldg(xr + q), m);
+      if ((k & m0) == p0) atomicAdd(&sm.hist[0][(k >> shift) & dm], 1u);
+      if (!same && (k & m1) == p1) atomicAdd(&sm.hist[1][(k >> shift) & dm], 1u);
+    }
+    os_scan(sm, shift, w, tid);
+    left = shift;
+  }
+  if (left == 0) return;
+  const unsigned p0 = sm.pfx[0], m0 = sm.mask[0], p1 = sm.pfx[1], m1 = sm.mask[1];
+  int n = 0;
+  for (int q = tid; q < T; q += kOsThreads) {
+    const unsigned k = os_key<kDev>(__ldg(xr + q), m);
+    if ((k & m0) == p0 || (k & m1) == p1) seg[n++] = k;
+  }
+  os_tail(seg, n, sm, left, tid);
 }
 
 // Row u of x (T values): the ka-th and kb-th largest, their keys to
@@ -246,9 +332,14 @@ __global__ void __launch_bounds__(kOsThreads, 1) order_stats_kernel(const float*
   const float* xr = x + (size_t)u * T;
   const int nv = max(0, min(kOsPer, T - tid * kOsPer));
   unsigned* seg = &sm.stage[tid * kOsSeg];
-  os_stage<false>(xr, T, 0.f, sm, tid);
-  __syncthreads();
-  os_select2(seg, nv, sm, ka, kb, tid);
+  const bool long_row = T > kOsThreads * kOsPer;
+  if (long_row) {
+    os_select2_long<false>(xr, T, 0.f, seg, sm, ka, kb, tid);
+  } else {
+    os_stage<false>(xr, T, 0.f, sm, tid);
+    __syncthreads();
+    os_select2(seg, nv, sm, ka, kb, tid);
+  }
   const unsigned a = sm.pfx[0], b = sm.pfx[1];
   if (tid == 0) {
     out[4 * u] = a;
@@ -259,9 +350,13 @@ __global__ void __launch_bounds__(kOsThreads, 1) order_stats_kernel(const float*
   // select reordered the stage)
   const float m = __fmul_rn(0.5f, __fadd_rn(key_float(a), key_float(b)));
   __syncthreads();  // every thread has read the first pair and its last list
-  os_stage<true>(xr, T, m, sm, tid);
-  __syncthreads();
-  os_select2(seg, nv, sm, ka, kb, tid);
+  if (long_row) {
+    os_select2_long<true>(xr, T, m, seg, sm, ka, kb, tid);
+  } else {
+    os_stage<true>(xr, T, m, sm, tid);
+    __syncthreads();
+    os_select2(seg, nv, sm, ka, kb, tid);
+  }
   if (tid == 0) {
     out[4 * (2 * rows + u)] = sm.pfx[0];
     out[4 * (3 * rows + u)] = sm.pfx[1];
@@ -272,7 +367,7 @@ __global__ void __launch_bounds__(kOsThreads, 1) order_stats_kernel(const float*
 
 cudaError_t launch_order_stats(const float* x, int rows, int T, int ka, int kb, bool mad, unsigned* out,
                                cudaStream_t s) {
-  if (rows <= 0 || T <= 0 || T > kOsThreads * kOsPer || ka < 1 || ka > T || kb < 1 || kb > T)
+  if (rows <= 0 || T <= 0 || T > kMaxN || ka < 1 || ka > T || kb < 1 || kb > T)
     return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)rows);

@@ -145,8 +145,7 @@ def test_wide_cluster_ragged(pool_kernel):
 
 
 # (32768, 8): the finalize takes clusters of four CTAs of 8192 candidates;
-# (65536, 4): more candidates than one thread-block cluster holds, so the
-# finalize runs one CTA per head
+# (65536, 4): clusters of eight such CTAs
 @pytest.mark.parametrize("n,window", [(1024, 1), (4096, 32), (16384, 4), (32768, 8), (65536, 4)])
 def test_sweep_points(n, window):
     run_and_compare(sweep_workload(n, window))
@@ -154,7 +153,7 @@ def test_sweep_points(n, window):
 
 def test_sweep_largest_point_sampled_heads():
     # the sweep's longest layer (131072 tokens, W = 16: g W = 64 rows on the
-    # tensor cores; 131056 candidates, so the one-CTA finalize), every head
+    # tensor cores; 131056 candidates, clusters of sixteen CTAs), every head
     # scored in one call, two heads against the oracle
     run_and_compare(sweep_workload(131072, 16), units=[(0, 0), (0, 5)])
 
@@ -310,8 +309,10 @@ def test_mad_scaling_c2_two_layers():
 # off by one moves s_E by ~1e-4
 @pytest.mark.parametrize("flags", [E.ECOKV_FLAG_WINSOR_5, E.ECOKV_FLAG_WINSOR_1, E.ECOKV_FLAG_MAD],
                          ids=["winsor5", "winsor1", "mad"])
-@pytest.mark.parametrize("n", [5000, 20001, 32768])
+@pytest.mark.parametrize("n", [5000, 20001, 32768, 40000, 131072])
 def test_robust_order_statistics_exact(flags, n):
+    # past 32768 candidates the rows are read from L2 until the keys under the
+    # ranks' prefixes fit the shared-memory slots
     w = small_workload(n, h_kv=2, group=4, window=8, budget=n // 10, dtype="bf16", clustered=True, seed=3)
     K, V, Q = make_inputs(w)
     p = params_of(w, flags=flags)

@@ -8,7 +8,7 @@ import torch
 
 from oracle import ecokv_oracle as O
 from paper_2609_06663_gb300 import ecokv as E
-from paper_2609_06663_gb300.workloads import make_inputs, small_workload, workload
+from paper_2609_06663_gb300.workloads import make_inputs, small_workload, sweep_workload, workload
 from tests.parity import TOL, check_rows, check_selection, oracle_params, score_error
 
 DEV = "cuda"
@@ -98,8 +98,37 @@ def test_value_norm_flag_changes_the_scores_and_is_refused_without_values():
 
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("n", [65536, 131072])
+@pytest.mark.parametrize("flags", [E.ECOKV_FLAG_VNORM_IMP, E.ECOKV_FLAG_WINSOR_5, E.ECOKV_FLAG_MAD],
+                         ids=["vnorm", "winsor5", "mad"])
+def test_variants_on_long_heads(flags, n):
+    # the sweep's long layers: clusters of 8 (65532 candidates) and 16 CTAs
+    # (131068) finalize the heads, and the order statistics read the rows
+    # from L2 instead of holding them in shared memory; two heads against the
+    # oracle
+    w = sweep_workload(n, 4)
+    K, V, Q = make_inputs(w)
+    p = params_of(w, flags)
+    idx, Ko, Vo, S, lam = E.evict(p, K.to(DEV), V.to(DEV), Q.to(DEV), want_scores=True)
+    torch.cuda.synchronize()
+    op = oracle_params(p)
+    units = [(0, 0), (0, 5)]
+    ref = O.evict(K, V, Q, op, heads=units)
+    tol = TOL[w.dtype]
+    S_np = S.cpu().double().numpy()
+    for (l, h) in units:
+        r = ref[(l, h)]
+        what = f"{w.name} unit ({l},{h}) flags {flags:#x}"
+        assert score_error(S_np[l, h], r["S"]) <= tol, what
+        assert abs(float(lam[l, h]) - r["lam"]) <= tol, what
+        check_selection(idx[l, h].cpu().numpy(), r, op, tol, what)
+        check_rows(V[l, h].to(DEV), idx[l, h], Vo[l, h], what)
+
+
+@pytest.mark.gpu
 def test_value_norm_refused_past_the_cluster_finalize():
-    w = small_workload(40000, h_kv=1, group=1, window=4, budget=400, dtype="bf16")
+    # past 16 x 8192 candidates no cluster shape takes the head
+    w = small_workload(140000, h_kv=1, group=1, window=4, budget=400, dtype="bf16")
     K, V, Q = make_inputs(w, device=DEV)
     with pytest.raises(E.EcokvError) as e:
         E.evict(params_of(w), K, V, Q)
