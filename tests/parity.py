@@ -64,3 +64,30 @@ def check_rows(K: torch.Tensor, idx: torch.Tensor, K_out: torch.Tensor, what="")
     """K_out[r] must be a bit-exact copy of K[idx[r]]."""
     ref = K[idx.long().cpu()] if K.device.type == "cpu" else K[idx.long()]
     assert torch.equal(K_out.to(ref.device), ref), f"{what}: compacted rows differ"
+
+
+# ---------------------------------------------------------------- canaries
+GUARD_BYTES = 256  # keeps the guarded view 16-byte aligned
+_CANARY = {torch.float32: float("nan"), torch.bfloat16: float("nan"), torch.int32: -0x5A5A5A5B}
+
+
+class Guarded:
+    """An output tensor with guard regions before and after it, filled with a
+    sentinel that no call may overwrite (out-of-bounds writes of the kernels
+    show up here, the sanitizer being unavailable)."""
+
+    def __init__(self, shape, dtype, device):
+        import math
+        self.g = GUARD_BYTES // torch.tensor([], dtype=dtype).element_size()
+        n = math.prod(shape)
+        self.full = torch.empty(n + 2 * self.g, dtype=dtype, device=device)
+        self.full.fill_(_CANARY[dtype])
+        self.view = self.full[self.g:self.g + n].view(*shape)
+        self.view.zero_()
+
+    def check(self, what=""):
+        for part in (self.full[:self.g], self.full[-self.g:]):
+            bits = part.view(torch.int16 if part.element_size() == 2 else torch.int32)
+            ref = torch.empty_like(part).fill_(_CANARY[part.dtype])
+            ref_bits = ref.view(torch.int16 if ref.element_size() == 2 else torch.int32)
+            assert torch.equal(bits, ref_bits), f"{what}: a guard region next to an output was overwritten"

@@ -11,7 +11,7 @@ import torch
 from oracle import ecokv_oracle as O
 from paper_2609_06663_gb300 import ecokv as E
 from paper_2609_06663_gb300.workloads import CONFIGS, make_inputs, small_workload, sweep_workload, workload
-from tests.parity import TOL, check_rows, check_scores, check_selection, oracle_params, score_error
+from tests.parity import TOL, Guarded, check_rows, check_scores, check_selection, oracle_params, score_error
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -30,11 +30,25 @@ def run_and_compare(w, layers=None, units=None, **kw):
     p = params_of(wl, **kw)
     Kd, Vd, Qd = K.to(DEV), V.to(DEV), Q.to(DEV)
     ws = E.alloc_workspace(p, DEV)
-    S, lam, dbg = E.score(p, Kd, Qd, ws=ws, dbg=True)
-    idx, Ko, Vo, S2, lam2 = E.evict(p, Kd, Vd, Qd, ws=ws, want_scores=True)
-    idx_sel = E.select(p, S)
+    # every output between guard regions (checked after the calls)
+    n_keep, tv = min(p.budget, p.n), p.n - p.window
+    dt = E.dtype_code(Kd)
+    g = {k: Guarded(shape, t, DEV) for k, (shape, t) in {
+        "S": ((nl, w.h_kv, tv), torch.float32), "lam": ((nl, w.h_kv), torch.float32),
+        "dbg": ((nl, w.h_kv, 5, tv), torch.float32), "idx": ((nl, w.h_kv, n_keep), torch.int32),
+        "Ko": ((nl, w.h_kv, n_keep, p.d), Kd.dtype), "Vo": ((nl, w.h_kv, n_keep, p.d), Kd.dtype),
+        "S2": ((nl, w.h_kv, tv), torch.float32), "lam2": ((nl, w.h_kv), torch.float32),
+        "idx_sel": ((nl, w.h_kv, n_keep), torch.int32)}.items()}
+    S, lam, dbg = g["S"].view, g["lam"].view, g["dbg"].view
+    idx, Ko, Vo, S2, lam2 = g["idx"].view, g["Ko"].view, g["Vo"].view, g["S2"].view, g["lam2"].view
+    idx_sel = g["idx_sel"].view
+    assert E.ecokv_score(p, dt, Kd, Qd, S, lam, dbg, ws, ws.numel()) == 0
+    assert E.ecokv_evict(p, dt, Kd, Vd, Qd, idx, Ko, Vo, S2, lam2, ws, ws.numel()) == 0
+    assert E.ecokv_select(p, S, idx_sel) == 0
     torch.cuda.synchronize()
     assert E.ecokv_device_status(ws) == 0
+    for k, gk in g.items():
+        gk.check(f"{w.name} {k}")
     # fused entry == split entries, bit for bit
     assert torch.equal(S, S2) and torch.equal(lam, lam2) and torch.equal(idx, idx_sel)
     op = oracle_params(p)
