@@ -1,8 +1,8 @@
 // Persistent tensor-core kernel for bf16 inputs: both streaming passes of the
 // eviction pass in one launch on sm_103a.
 //
-// Work items (u = unit = (layer, KV head); a chunk is up to 64 tiles of 128
-// consecutive keys of one unit):
+// Work items (u = unit = (layer, KV head); a chunk is a run of consecutive
+// tiles of 128 keys of one unit, the part of a CTA's slice inside the unit):
 //   P1(u, c)  pass 1 over chunk c: window logits (tcgen05 MMA, keys as M,
 //             window rows as N), per-row online-softmax partials, key norms,
 //             and the chunk sums of k and k/||k|| (a second tcgen05 MMA with the
@@ -16,38 +16,44 @@
 //             of ||k||^2 + ||kbar||^2, keys close to their centroid) the key is
 //             recomputed directly from its row in global memory.
 //
-// Schedule.  The chunks of all units, in unit order, form blocks of `blk`
-// chunks.  Tickets, taken from a global counter, run through steps: step s
-// holds the P1 items of block s, then the P2 items of block s - lag.  Pass 2
-// of a chunk therefore follows its pass 1 by about lag blocks of DRAM reads,
-// which the host keeps well inside L2: the second read of every key hits L2,
-// so K crosses the HBM interface once.  Every item depends only on items with
-// smaller tickets, so dispatch is deadlock-free without co-residency.  The
-// last P2 items may be split in parts (each with its own partial slot), so
-// that the CTAs run out of work together.
+// Schedule (static, one CTA per SM, cooperative launch).  The units form
+// waves of `uw` units in unit order; the tiles of a wave are cut into
+// n = min(P, L) contiguous slices of near-equal length (L = the wave's
+// tiles), and CTA c takes slice c of every wave, one item per unit the slice
+// touches.  Step s of CTA c holds: the P1 items of its slice of wave s; the
+// fold items of the units of wave s - 1 it owns (unit u belongs to CTA
+// u mod P); the P2 items of its slice of wave s - lag.  With one wave (the
+// default) all of pass 1 precedes pass 2 and K is read twice; with small
+// waves and lag 1..2 a unit's keys are still in L2 at its pass 2 (pass-1
+// reads carry an evict-last policy then), at the cost of more items.  Every
+// CTA is resident, so waits on other CTAs' items end.
 //
-// Unit statistics (kbar, mu, ||kbar||^2, ||mu||^2, per-row log2-sum-exp): the
-// first CTA to start a P2 item of unit u claims the unit (an atomic on a
-// per-unit word); its epilogue warps wait until every P1 item of u has
-// arrived (a per-unit counter the stats warp of each CTA increments with
-// release semantics), fold the chunk partials in a fixed order with all 256
-// threads, publish the record and raise the unit's ready flag.  Other P2
-// items of u wait for that flag and read the record.  Nothing but the MMA and
-// the epilogue of a P2 item waits for it: the producer keeps loading key
-// tiles meanwhile.
+// Unit statistics (kbar, mu, ||kbar||^2, ||mu||^2, per-row log2-sum-exp):
+// every P1 item writes a record to its slot (its slice's index among the
+// slices the unit meets) and then adds one to the unit's arrival counter with
+// release semantics.  The fold item of unit u waits until all of the unit's
+// slices have arrived, folds the records in a fixed order with the 256
+// epilogue threads, publishes the statistics record and raises the unit's
+// ready flag (release).  The stats warp readies each P2 item about one item
+// ahead of the epilogue: it waits for the flag, copies the record and writes
+// the statistics rows of the MMA operand.  Nothing but the MMA and the
+// epilogue of a P2 item waits for it: the producer keeps loading key tiles
+// meanwhile.  The fold order and every partial's arithmetic depend only on
+// the schedule's parameters, so results are reproducible for a given
+// (uw, lag, P).
 //
-// Warp roles (512 threads, one CTA per SM): warp 0 takes tickets and issues
-// TMA loads of the window queries and of 32 KB key tiles into a 5-stage ring;
-// warp 1 issues the logits MMAs into up to four TMEM accumulators; warp 3
-// issues the sum MMAs of pass-1 tiles (two more accumulators) as soon as a
-// tile's logits are done and its weights written, and frees the stage; warp 2
-// counts finished pass-1 items per unit; warps 12-15 (key warps, one key per
-// thread) compute the key norms of every tile as it lands (the sum weights in
-// pass 1, a hand-off to the epilogue in pass 2) and read the chunk sums;
-// warps 4-11 are the epilogue (one key per TMEM lane, window rows split in two
-// halves), which also folds or reads the unit statistics and writes the
-// statistics rows of the MMA operand at the start of a P2 item.  setmaxnreg
-// gives the two epilogue warpgroups 176 registers a thread and the others 80.
+// Warp roles (512 threads, one CTA per SM): warp 0 walks the CTA's schedule
+// and issues TMA loads of the window queries and of 32 KB key tiles into a
+// 4- or 5-stage ring; warp 1 issues the logits MMAs into up to four TMEM
+// accumulators; warp 3 issues the sum MMAs of pass-1 tiles (two more
+// accumulators) as soon as a tile's logits are done and its weights written,
+// and frees the stage; warp 2 (stats warp) readies the unit statistics of P2
+// items; warps 12-15 (key warps, one key per thread) compute the key norms of
+// every tile as it lands (the sum weights in pass 1, a hand-off to the
+// epilogue in pass 2) and read the chunk sums; warps 4-11 are the epilogue
+// (one key per TMEM lane, window rows split in two halves), which also runs
+// the fold items.  setmaxnreg gives the two epilogue warpgroups 176
+// registers a thread and the others 80.
 // Every mbarrier wait and spin is bounded (a limit in nanoseconds of the
 // global timer): on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
 // gpu-wide abort flag, drains its own copies (key tiles and window queries)
@@ -1063,8 +1069,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         part[kk] = __uint_as_float(v[0]);
         part[kD + kk] = (__uint_as_float(v[1]) + __uint_as_float(v[2])) + __uint_as_float(v[3]);
       }
-      // the item's key norms and sums are written: the stats warp's gpu-scope
-      // arrival (after it has waited for kpub) publishes them
+      // the item's chunk sums are written: the epilogue's gpu-scope arrival
+      // (after it has waited for kpub) publishes them
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&s.kpub[slot]);
