@@ -20,7 +20,8 @@
 // waves of `uw` units in unit order; the tiles of a wave are cut into
 // n = min(P, L) contiguous slices of near-equal length (L = the wave's
 // tiles), and CTA c takes slice c of every wave, one item per unit the slice
-// touches.  Step s of CTA c holds: the P1 items of its slice of wave s; the
+// touches (pass 2 walks a slice backwards, units and tiles, so that it starts
+// with the keys pass 1 read last, the likeliest still to be in L2).  Step s of CTA c holds: the P1 items of its slice of wave s; the
 // fold items of the units of wave s - 1 it owns (unit u belongs to CTA
 // u mod P); the P2 items of its slice of wave s - lag.  With one wave (the
 // default) all of pass 1 precedes pass 2 and K is read twice; with small
@@ -604,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float ksq = d.ust[ustat_ksq()];
         float s_all = 0.f, mn = INFINITY, mx = -INFINITY, s_de = 0.f, s_c = 0.f, s_raw = 0.f;
         for (int t = 0; t < ntiles && ok; ++t) {
-          const int i = i0 + t * kTile + kk;
+          const int i = i0 + (ntiles - 1 - t) * kTile + kk;  // pass 2 walks the item backwards
           const bool valid = i < a.N;
           const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.tmem_full[b], tph, a, 14u)))) break;
@@ -783,7 +784,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           good = wait_bar(&s.empty[stage], sphase ^ 1u, a, 4u);
           if (good) {
             mbar_expect_tx(&s.full[stage], kTileBytes);
-            const int y = i0 + t * kTile;
+            const int y = i0 + (type == kP2 ? ntiles - 1 - t : t) * kTile;
             tma_load_3d_hint(s.ktile[stage], &tmK, &s.full[stage], 0, y, u, pol);
             tma_load_3d_hint(s.ktile[stage] + kTileBytes / 2, &tmK, &s.full[stage], 64, y, u, pol);
             used_bits |= 1u << stage;
@@ -819,7 +820,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c >= n) continue;
         const int g0 = w * a.uw * a.T;  // the wave's first tile, counted over all units
         const int lo = g0 + slice_start(c, L, n), hi = g0 + slice_start(c + 1, L, n);
-        for (int u = lo / a.T; u * a.T < hi && ok; ++u) {
+        // pass 2 walks the slice backwards (units and tiles): the keys pass 1
+        // read last are the likeliest still to be in L2
+        const int u_first = lo / a.T, u_last = (hi - 1) / a.T;
+        for (int k = 0; u_first + k <= u_last && ok; ++k) {
+          const int u = ph == 0 ? u_first + k : u_last - k;
           const int t_lo = max(lo, u * a.T) - u * a.T, t_hi = min(hi, (u + 1) * a.T) - u * a.T;
           int c0, nrec;
           unit_slices(a, u, c0, nrec);
@@ -1001,7 +1006,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (type == kExit) break;
       for (int t = 0; t < ntiles && ok; ++t) {
         if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.full[stage], sphase, a, 22u)))) break;
-        const int i = i0 + t * kTile + kk;
+        const int i = i0 + (type == kP2 ? ntiles - 1 - t : t) * kTile + kk;
         const bool valid = i < a.N;
         // squared norm of this thread's key (packed fp32 pairs), the same
         // arithmetic in both passes
