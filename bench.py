@@ -87,15 +87,23 @@ def byte_model(w) -> dict:
     return {"alg": alg, "bl": bl, "k": k_bytes, "q": q_bytes, "kept_rows": kept}
 
 
+def tensor_path(w) -> bool:
+    """bf16 inputs of at least 128 keys stream through the tensor-core kernel."""
+    return w.dtype == "bf16" and w.n >= 128
+
+
+def row_groups(w) -> int:
+    """Launches of the tensor-core kernel per call: one per group of at most
+    120 window rows (g * W rows per head)."""
+    return (w.group * w.window + 119) // 120
+
+
 def launches_per_call(w) -> int:
     """Kernels one ecokv_evict call launches: the persistent tensor-core
-    streaming kernel (bf16, n >= 128, padded g*W + 8 statistics rows <= 128)
-    or the two CUDA-core passes, then the finalize/select kernel (one thread-
-    block cluster per head, or one CTA per head past 32768 candidates) and the
-    compaction kernel."""
-    r = w.group * w.window
-    tc = w.dtype == "bf16" and w.n >= 128 and ((r + 3) // 4) * 4 + 8 <= 128
-    return (1 if tc else 2) + 2
+    streaming kernel (once per window-row group) or the two CUDA-core passes,
+    then the finalize/select kernel (one thread-block cluster per head, or one
+    CTA per head past 131072 candidates) and the compaction kernel."""
+    return (row_groups(w) if tensor_path(w) else 2) + 2
 
 
 # ---------------------------------------------------------------- ranks
@@ -468,7 +476,7 @@ def main():
     bm = byte_model(w)
     peak, peak_kind = measured_peaks()
     tr = traffic_record(args.workload)
-    tc = launches_per_call(w) == 3
+    tc = tensor_path(w)
     # dominant kernel: the streaming pass; its algorithmic bytes are every K
     # row and the window queries read once
     stream_bytes = bm["k"] + bm["q"]
@@ -589,7 +597,7 @@ def run_sweep(args) -> None:
             print(json.dumps({
                 "sweep": "bandwidth sweep (one layer, 8 KV / 32 query heads, bf16, budget 10 %)",
                 "workload": w.name, "n": n, "window": win, "budget": w.budget,
-                "path": "tensor-core streaming kernel" if launches_per_call(w) == 3 else "CUDA-core passes",
+                "path": (f"tensor-core streaming kernel x{row_groups(w)}" if tensor_path(w) else "CUDA-core passes"),
                 "ms_per_call": round(ms, 5), "tokens_per_s": round(w.units * n / (ms * 1e-3), 1),
                 "evicted_rows_per_s": round(w.units * max(0, n - w.budget) / (ms * 1e-3), 1),
                 "alg_gbs": round(gbs(bm["alg"], ms), 1), "bl_gbs": round(gbs(bm["bl"], ms), 1),

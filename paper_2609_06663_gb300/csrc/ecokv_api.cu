@@ -2,8 +2,9 @@
 // launches.  Every entry point validates on the host and returns before
 // launching anything when an argument is wrong.
 //
-// Paths.  bf16 inputs with n >= 128 and (h_q/h_kv)*W <= 120 stream K through
-// the persistent tensor-core kernel (tc_pass.cu, one launch for both passes);
+// Paths.  bf16 inputs with n >= 128 stream K through the persistent
+// tensor-core kernel (tc_pass.cu, one launch for both passes, or one launch
+// per group of at most 120 window rows when (h_q/h_kv)*W exceeds 120);
 // fp32 inputs, other shapes and calls with ECOKV_FLAG_FORCE_SIMT use the
 // CUDA-core passes (score_simt.cu, two launches).  Either way one more launch
 // (finalize_select.cu) turns the pass-2 outputs into scores, selects and
@@ -69,10 +70,16 @@ static ecokv_status check_ws(const ecokv_params* p, void* ws, size_t ws_bytes) {
   return ECOKV_OK;
 }
 
+// Window rows per launch of the tensor-core kernel: all R of a unit when
+// R <= 120 (the MMA's N holds the rows padded to four plus eight statistics
+// columns, at most 128), else R split into ceil(R / 120) near-equal groups.
+static int tc_groups(int R) { return (R + 119) / 120; }
+static int tc_group_rows(int R) { return (R + tc_groups(R) - 1) / tc_groups(R); }
+
 static bool use_tensor_path(const ecokv_params& p, ecokv_dtype dt) {
   if (dt != ECOKV_BF16 || (p.flags & ECOKV_FLAG_FORCE_SIMT)) return false;
   if (p.n < 128) return false;
-  return tc_rows_half((p.h_q / p.h_kv) * p.window) > 0;
+  return tc_rows_half(tc_group_rows((p.h_q / p.h_kv) * p.window)) > 0;
 }
 
 // Stage events of this host thread (ecokv_set_stage_events), recorded on the
@@ -199,17 +206,35 @@ static unsigned long long wait_limit_ns(const ecokv_params& p) {
 }
 
 // Both streaming passes on the tensor cores in one launch (after clearing
-// the per-call counters).
+// the per-call counters), or one launch per window-row group: pass 1 of a
+// group gives its rows' log-sum-exp (the centroid sums are the same in every
+// group), pass 2 adds the group's vote to the vote of the groups before it.
+// Every group reads K twice.
+static ecokv_status run_tc_group(const ecokv_params& p, const Layout& L, const void* K, const void* Q, char* ws,
+                                 int row0, int rows, int rows_max, cudaStream_t s);
+
 static ecokv_status run_tc_passes(const ecokv_params& p, const void* K, const void* Q, char* ws, cudaStream_t s) {
   const Layout L = make_layout(p, tc_records(p));
+  const int Rg = tc_group_rows(L.R);
+  for (int row0 = 0; row0 < L.R; row0 += Rg) {
+    const int rows = L.R - row0 < Rg ? L.R - row0 : Rg;
+    const ecokv_status st = run_tc_group(p, L, K, Q, ws, row0, rows, Rg, s);
+    if (st != ECOKV_OK) return st;
+  }
+  return ECOKV_OK;
+}
+
+static ecokv_status run_tc_group(const ecokv_params& p, const Layout& L, const void* K, const void* Q, char* ws,
+                                 int row0, int rows, int rows_max, cudaStream_t s) {
   if (cudaMemsetAsync(ws + L.sync, 0, L.sync_bytes, s) != cudaSuccess) return ECOKV_ERR_CUDA;
   TcArgs a{};
   a.U = L.U;
   a.N = p.n;
   a.W = p.window;
-  a.R = L.R;
-  a.R4 = (L.R + 3) & ~3;
-  a.NP = 2 * tc_rows_half(L.R);
+  a.R = rows;
+  a.R4 = (rows + 3) & ~3;
+  a.row0 = row0;
+  a.NP = 2 * tc_rows_half(rows_max);
   a.g = p.h_q / p.h_kv;
   a.h_kv = p.h_kv;
   a.h_q = p.h_q;

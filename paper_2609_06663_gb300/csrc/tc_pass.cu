@@ -334,7 +334,7 @@ __device__ void fold_unit_stats(const TcArgs& a, int u, int nch, int tid, float*
       const float m2 = s_fold[2 * (gg * R + tid)], z2 = s_fold[2 * (gg * R + tid) + 1];
       if (z2 > 0.f) combine_maxsum(Mx, Zx, m2, z2);
     }
-    gus[ustat_lse() + tid] = Mx + log2f(Zx);
+    gus[ustat_lse() + a.row0 + tid] = Mx + log2f(Zx);
   }
 }
 
@@ -509,7 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool full_vis = it0 + kTile - 1 <= a.N - a.W;  // every window row sees every key
           const int vis_from = i - (a.N - a.W);                 // else row j sees key i iff j >= vis_from
           if (t == 0) {
-            int j = (h * RH) % a.W;
+            int j = (a.row0 + h * RH) % a.W;  // the window position of the half's first row
 #pragma unroll
             for (int c = 0; c < RH; ++c) {
               const bool vis = full_vis || (valid && j >= vis_from);
@@ -527,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mx = fmaxf(mx, dl);
               }
             } else {
-              int j = (h * RH) % a.W;
+              int j = (a.row0 + h * RH) % a.W;  // the window position of the half's first row
 #pragma unroll
               for (int c = 0; c < RH; ++c) {
                 const bool vis = valid && j >= vis_from;
@@ -674,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 s_c += cs;
                 s_raw += v;
                 const size_t o = (size_t)u * a.Tv + i;
-                a.simp[o] = v;
+                a.simp[o] = a.row0 == 0 ? v : __ldcg(a.simp + o) + v;
                 a.dE[o] = dEv;
                 a.cosv[o] = cs;
               }
@@ -716,7 +716,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the item's record slot; the unit's first record also fills every
           // slot past the unit's records with the identity of its reduction
           float* p = a.p2part + (size_t)u * a.rmax * kP2Stride;
-          p[rec * kP2Stride + tid] = acc;  // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW
+          // P2_SUM_DE_ALL, P2_MIN_DE, P2_MAX_DE, P2_SUM_DE, P2_SUM_COS, P2_SUM_RAW; a later row group
+          // adds its vote sum, the distance and cosine partials are the same in every group
+          if (tid == P2_SUM_RAW && a.row0 > 0) acc += __ldcg(p + rec * kP2Stride + tid);
+          p[rec * kP2Stride + tid] = acc;
           if (rec == 0) {
             int c0, nrec;
             unit_slices(a, u, c0, nrec);
@@ -768,7 +771,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // window queries by TMA (swizzled in flight); the MMA (pass 1) or
           // the stats warp (pass 2) waits for them, not this warp
           const int layer = u / a.h_kv, head = u % a.h_kv;
-          const int qrow = (layer * a.h_q + head * a.g) * a.W;
+          const int qrow = (layer * a.h_q + head * a.g) * a.W + a.row0;
           mbar_expect_tx(&s.qfull[slot], (uint32_t)a.NP * 256u);
           tma_load_2d(s.qbuf[slot], &tmQ, &s.qfull[slot], 0, qrow);
           tma_load_2d(s.qbuf[slot] + a.NP * 128, &tmQ, &s.qfull[slot], 64, qrow);
@@ -980,9 +983,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         __syncwarp();  // lane 0's acquire orders the record's loads below
         const float4* g = reinterpret_cast<const float4*>(a.ustat + (size_t)u * a.ustat_stride);
-        for (int e4 = lane; e4 < a.ustat_stride / 4; e4 += 32) reinterpret_cast<float4*>(ust)[e4] = __ldcg(g + e4);
-        __syncwarp();
-        for (int r = a.R + lane; r < a.NP; r += 32) ust[ustat_lse() + r] = INFINITY;
+        for (int e4 = lane; e4 < ustat_lse() / 4; e4 += 32) reinterpret_cast<float4*>(ust)[e4] = __ldcg(g + e4);
+        // this row group's log2-sum-exp rows; +inf past them
+        const float* gl = a.ustat + (size_t)u * a.ustat_stride + ustat_lse() + a.row0;
+        for (int r = lane; r < a.NP; r += 32) ust[ustat_lse() + r] = r < a.R ? __ldcg(gl + r) : INFINITY;
         if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.qfull[slot], ((qpar >> slot) & 1u) ^ 1u, a, 27u)))) break;
         for (int e = lane; e < 5 * 16; e += 32) build_stat_rows(s.qbuf[slot], a, ust, e);
         fence_proxy_async_smem();

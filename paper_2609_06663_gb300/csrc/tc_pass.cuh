@@ -8,7 +8,8 @@ namespace ecokv {
 constexpr int kTcMaxSms = 256;                 // largest grid the record slots are sized for
 
 struct TcArgs {
-  int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;
+  int U, N, W, R, R4, NP, g, h_kv, h_q, Tv;  // R, R4: rows of this launch's row group
+  int row0;                         // the group's first window row among the unit's (h_q / h_kv) * W
   int kbar_n;                       // keys 0 .. kbar_n - 1 form the centroid (N, or Tv for the non-window centroid)
   int q_rows;                       // rows of the window-query tensor: n_layers * h_q * W
   int T;                            // tiles of 128 keys per unit: ceil(N / 128)

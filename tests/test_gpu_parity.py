@@ -90,6 +90,10 @@ SMALL = [
     dict(n=2, h_kv=1, group=3, window=1, budget=1, pool_kernel=3, dtype="bf16"),
     dict(n=5000, h_kv=2, group=7, window=8, budget=500, pool_kernel=5, dtype="bf16", n_layers=2,
          clustered=True),
+    # more window rows than one launch of the tensor-core kernel holds (120):
+    # g W = 224 in two row groups of 112, g W = 240 in two of 120
+    dict(n=3000, h_kv=2, group=7, window=32, budget=300, pool_kernel=5, dtype="bf16", clustered=True),
+    dict(n=1500, h_kv=1, group=8, window=30, budget=200, pool_kernel=5, dtype="bf16"),
 ]
 
 
@@ -113,6 +117,14 @@ def test_streaming_schedules(wave, lag):
     w = small_workload(5000, h_kv=2, group=7, window=8, budget=500, pool_kernel=5, dtype="bf16", n_layers=3,
                        clustered=True)
     run_and_compare(w, sched_wave=wave, sched_lag=lag)
+
+
+def test_streaming_schedule_row_groups():
+    """Two window-row groups (g W = 128) with waves of one head: each group's
+    pass 2 adds its vote to the earlier group's."""
+    w = small_workload(3000, h_kv=2, group=8, window=16, budget=300, pool_kernel=5, dtype="bf16", n_layers=2,
+                       clustered=True)
+    run_and_compare(w, sched_wave=1, sched_lag=1)
 
 
 def test_streaming_schedule_many_units():
