@@ -40,6 +40,14 @@
  *    in the workspace's status word; read them with ecokv_device_status().
  *  - Calls that share a workspace must be ordered on one stream.
  *  - Inputs must be finite; scores of non-finite inputs are unspecified.
+ *  - Paths: bf16 inputs with n >= 128 stream K through a persistent
+ *    tensor-core kernel, one launch for both of its passes over K, or one
+ *    launch per group of at most 120 window rows when (h_q / h_kv) * window
+ *    exceeds 120 (each group reads K twice); fp32 inputs, shorter caches and
+ *    ECOKV_FLAG_FORCE_SIMT take the CUDA-core passes.  Every path is
+ *    deterministic; scores may differ in their last bits between paths and
+ *    between streaming schedules (ecokv_params.sched_*), within the
+ *    documented tolerances.
  */
 #ifndef ECOKV_H
 #define ECOKV_H
