@@ -114,9 +114,8 @@ struct __align__(1024) Smem {
   uint8_t qbuf[kIQ][kQB < 1024 ? 1024 : kQB];   // B operand, 2 boxes [NP rows x 64 d]
   uint8_t wbuf[kS][4096];                       // sum weights: 2 boxes [16 rows x 64 keys]; rows 1, w_hi, w_mid, w_lo
   ItemDesc desc[kIQ];
-  float xch[kNB][kTile];                        // pass-2 vote of the first row half, per key
   float red[8][RH][2];                          // [epilogue warp][row][max, sum]
-  float red6[4][8];                             // [second-half warp][pass-2 partial]
+  float red6[8][8];                             // [epilogue warp][pass-2 partial]
   uint64_t full[kS], empty[kS], wready[kS];
   uint64_t item_full[kIQ], item_empty[kIQ], qfull[kIQ];
   uint64_t tmem_full[4], tmem_empty[4];
@@ -124,7 +123,6 @@ struct __align__(1024) Smem {
   uint64_t lgdone[kS];  // pass-1 tile: its logits MMA is complete (for the sum-MMA issuer)
   float nbuf[kNB][kTile];                        // pass-2 squared key norms, key warps -> epilogue
   uint64_t nfull[kNB], nempty[kNB];
-  uint64_t xfull[kNB], xempty[kNB];             // first row half -> second row half, per pass-2 tile
   uint64_t kpub[kIQ];    // key warps have written this pass-1 item's chunk sums
   uint64_t sready[kIQ];  // pass 2: unit statistics in desc.ust and statistics rows in qbuf (stats warp ->
                          // MMA and epilogue)
@@ -398,9 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < kIQ; ++i) mbar_init(&s.kpub[i], kKeyWarps);
     for (int i = 0; i < kNB; ++i) {
       mbar_init(&s.nfull[i], kKeyWarps);
-      mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the second row half
-      mbar_init(&s.xfull[i], 4);   // first row half
-      mbar_init(&s.xempty[i], 4);  // second row half
+      mbar_init(&s.nempty[i], 4);  // the 4 epilogue warps of the half that takes the tile
     }
     s.epi_abort = 0;
     mbar_init(&s.drain, 1);
@@ -596,111 +592,120 @@ __global__ void __launch_bounds__(kThreads, 1)
           else s.epi_abort = 1;
         }
       } else {  // kP2
-        // the stats warp has copied the unit statistics and built the
-        // statistics rows
+        // Pass 2 splits the tiles, not the rows: the warps of row half h take
+        // the tiles t of the item with t % 2 == h and every row of them, so
+        // no warp waits for another within a tile and the two halves work on
+        // consecutive tiles at once.  Within an item a TMEM buffer (tcount
+        // mod 4 or 2) and a norm slot (tile mod kNB) always serve the same
+        // half; at item boundaries every epilogue warp meets at the item's
+        // first barrier, so a half never waits on a phase whose previous
+        // use the other half has not consumed.  The stats warp has copied
+        // the unit statistics and built the statistics rows.
         ok = __all_sync(0xffffffffu, wait_bar(&s.sready[slot], (spar >> slot) & 1u, a, 18u));
         spar ^= 1u << slot;
-        const float* lse = d.ust + ustat_lse();
         const float* kbv = d.ust + ustat_kbar();
         const float ksq = d.ust[ustat_ksq()];
+        // log2-sum-exp of every row (+inf past R: those vote terms, padding
+        // and statistics columns, are exactly zero), in registers unless the
+        // rows are too many; the tile's accumulator columns are read in
+        // chunks of kCW
+        constexpr int kCW = RH <= 32 ? 2 * RH : RH;
+        constexpr bool kLseReg = RH <= 32;
+        float lse_r[kLseReg ? 2 * RH : 1];
+#pragma unroll
+        for (int c = 0; c < (kLseReg ? 2 * RH : 1); ++c) lse_r[c] = d.ust[ustat_lse() + c];
+        const float* lse_s = d.ust + ustat_lse();
         float s_all = 0.f, mn = INFINITY, mx = -INFINITY, s_de = 0.f, s_c = 0.f, s_raw = 0.f;
         for (int t = 0; t < ntiles && ok; ++t) {
+          const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
+          const uint32_t ps = pcount % kNB, pph = (pcount / kNB) & 1u;
+          ++tcount;
+          ++pcount;
+          if ((t & 1) != h) continue;
           const int i = i0 + (ntiles - 1 - t) * kTile + kk;  // pass 2 walks the item backwards
           const bool valid = i < a.N;
-          const uint32_t b = tcount & bmask, tph = (tcount >> nbuf_log) & 1u;
           if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.tmem_full[b], tph, a, 14u)))) break;
           tc_fence_after();
-          uint32_t rc[RH];
-          tmem_ld<RH>(tl + b * (uint32_t)a.NP + (uint32_t)(h * RH), rc);
-          tmem_wait_ld();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.tmem_empty[b]);
-          ++tcount;
-          const uint32_t ps = pcount % kNB, pph = (pcount / kNB) & 1u;
-          ++pcount;
-          // vote of this half's rows; the lse of rows past R is +inf, so
-          // padding and statistics columns add exactly zero
-          float vp[4] = {0.f, 0.f, 0.f, 0.f};
+          // the vote of every row, chunk by chunk; the statistics columns
+          // are the last eight of the accumulator: k . kbar in three terms,
+          // k . mu in two
+          float vp[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          float kkb = 0.f, kmu = 0.f;
 #pragma unroll
-          for (int c = 0; c < RH; ++c) vp[c & 3] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -lse[h * RH + c]));
-          const float vh = (vp[0] + vp[1]) + (vp[2] + vp[3]);
-          if (h == 0) {
-            // hand the first half's vote to the second half
-            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.xempty[ps], pph ^ 1u, a, 24u)))) break;
-            s.xch[ps][kk] = vh;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.xfull[ps]);
-          } else {
-            // the statistics columns (the last eight of the accumulator):
-            // k . kbar in three terms, k . mu in two
-            const float kkb =
-                (__uint_as_float(rc[RH - 8]) + __uint_as_float(rc[RH - 7])) + __uint_as_float(rc[RH - 6]);
-            const float kmu = __uint_as_float(rc[RH - 5]) + __uint_as_float(rc[RH - 4]);
-            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nfull[ps], pph, a, 15u)))) break;
-            const float n2 = s.nbuf[ps][kk];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.nempty[ps]);
-            float d2 = fmaf(-2.f, kkb, n2) + ksq;
-            if (valid && d2 < 0.015625f * (n2 + ksq)) {
-              // cancellation regime: recompute |k - kbar|^2 from the key row
-              const uint4* row = reinterpret_cast<const uint4*>(a.K) + ((size_t)u * a.N + i) * 16;
-              float dp[4] = {0.f, 0.f, 0.f, 0.f};
-              for (int c = 0; c < 16; ++c) {
-                const uint4 kv = __ldg(row + c);
-                const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
-#pragma unroll
-                for (int t2 = 0; t2 < 4; ++t2) {
-                  const float dl = __uint_as_float(w4[t2] << 16) - kbv[c * 8 + 2 * t2];
-                  const float dh = __uint_as_float(w4[t2] & 0xffff0000u) - kbv[c * 8 + 2 * t2 + 1];
-                  dp[t2] = fmaf(dl, dl, dp[t2]);
-                  dp[t2] = fmaf(dh, dh, dp[t2]);
-                }
-              }
-              d2 = (dp[0] + dp[1]) + (dp[2] + dp[3]);
+          for (int c0 = 0; c0 < 2 * RH; c0 += kCW) {
+            uint32_t rc[kCW];
+            tmem_ld<kCW>(tl + b * (uint32_t)a.NP + (uint32_t)c0, rc);
+            tmem_wait_ld();
+            if (c0 + kCW == 2 * RH) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive_cnt(&s.tmem_empty[b], 2u);  // this half's four warps stand for all eight
+              kkb = (__uint_as_float(rc[kCW - 8]) + __uint_as_float(rc[kCW - 7])) + __uint_as_float(rc[kCW - 6]);
+              kmu = __uint_as_float(rc[kCW - 5]) + __uint_as_float(rc[kCW - 4]);
             }
-            const float dEv = sqrtf(fmaxf(d2, 0.f));
-            const float cs = kmu * rsqrtf(fmaxf(n2, 1e-24f));
-            if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.xfull[ps], pph, a, 25u)))) break;
-            const float v = vh + s.xch[ps][kk];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.xempty[ps]);
-            if (valid) {
-              s_all += dEv;
-              if (i < a.Tv) {
-                mn = fminf(mn, dEv);
-                mx = fmaxf(mx, dEv);
-                s_de += dEv;
-                s_c += cs;
-                s_raw += v;
-                const size_t o = (size_t)u * a.Tv + i;
-                a.simp[o] = a.row0 == 0 ? v : __ldcg(a.simp + o) + v;
-                a.dE[o] = dEv;
-                a.cosv[o] = cs;
+#pragma unroll
+            for (int c = 0; c < kCW; ++c)
+              vp[c & 7] += ex2(fmaf(__uint_as_float(rc[c]), a.scale_log2, -(kLseReg ? lse_r[c0 + c] : lse_s[c0 + c])));
+          }
+          const float v = ((vp[0] + vp[1]) + (vp[2] + vp[3])) + ((vp[4] + vp[5]) + (vp[6] + vp[7]));
+          // the key's squared norm from the key warps
+          if (!(ok = __all_sync(0xffffffffu, wait_bar(&s.nfull[ps], pph, a, 15u)))) break;
+          const float n2 = s.nbuf[ps][kk];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s.nempty[ps]);
+          float d2 = fmaf(-2.f, kkb, n2) + ksq;
+          if (valid && d2 < 0.015625f * (n2 + ksq)) {
+            // cancellation regime: recompute |k - kbar|^2 from the key row
+            const uint4* row = reinterpret_cast<const uint4*>(a.K) + ((size_t)u * a.N + i) * 16;
+            float dp[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int c = 0; c < 16; ++c) {
+              const uint4 kv = __ldg(row + c);
+              const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+              for (int t2 = 0; t2 < 4; ++t2) {
+                const float dl = __uint_as_float(w4[t2] << 16) - kbv[c * 8 + 2 * t2];
+                const float dh = __uint_as_float(w4[t2] & 0xffff0000u) - kbv[c * 8 + 2 * t2 + 1];
+                dp[t2] = fmaf(dl, dl, dp[t2]);
+                dp[t2] = fmaf(dh, dh, dp[t2]);
               }
+            }
+            d2 = (dp[0] + dp[1]) + (dp[2] + dp[3]);
+          }
+          const float dEv = sqrtf(fmaxf(d2, 0.f));
+          const float cs = kmu * rsqrtf(fmaxf(n2, 1e-24f));
+          if (valid) {
+            s_all += dEv;
+            if (i < a.Tv) {
+              mn = fminf(mn, dEv);
+              mx = fmaxf(mx, dEv);
+              s_de += dEv;
+              s_c += cs;
+              s_raw += v;
+              const size_t o = (size_t)u * a.Tv + i;
+              a.simp[o] = a.row0 == 0 ? v : __ldcg(a.simp + o) + v;
+              a.dE[o] = dEv;
+              a.cosv[o] = cs;
             }
           }
         }
-        // the chunk's six partials: warp butterflies in the second half, then
-        // its first warp combines the four warps in a fixed order
-        if (h == 1) {
+        // the chunk's six partials: warp butterflies, then one thread per
+        // partial combines the eight warps in a fixed order
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            s_all += __shfl_xor_sync(0xffffffffu, s_all, o);
-            mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            s_de += __shfl_xor_sync(0xffffffffu, s_de, o);
-            s_c += __shfl_xor_sync(0xffffffffu, s_c, o);
-            s_raw += __shfl_xor_sync(0xffffffffu, s_raw, o);
-          }
-          if (lane == 0) {
-            s.red6[e - 4][0] = s_all;
-            s.red6[e - 4][1] = mn;
-            s.red6[e - 4][2] = mx;
-            s.red6[e - 4][3] = s_de;
-            s.red6[e - 4][4] = s_c;
-            s.red6[e - 4][5] = s_raw;
-          }
+        for (int o = 16; o > 0; o >>= 1) {
+          s_all += __shfl_xor_sync(0xffffffffu, s_all, o);
+          mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+          s_de += __shfl_xor_sync(0xffffffffu, s_de, o);
+          s_c += __shfl_xor_sync(0xffffffffu, s_c, o);
+          s_raw += __shfl_xor_sync(0xffffffffu, s_raw, o);
+        }
+        if (lane == 0) {
+          s.red6[e][0] = s_all;
+          s.red6[e][1] = mn;
+          s.red6[e][2] = mx;
+          s.red6[e][3] = s_de;
+          s.red6[e][4] = s_c;
+          s.red6[e][5] = s_raw;
         }
         if (!epi_sync()) {
           ok = false;
@@ -709,8 +714,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (tid < 6) {
           float acc = s.red6[0][tid];
 #pragma unroll
-          for (int w4 = 1; w4 < 4; ++w4) {
-            const float x = s.red6[w4][tid];
+          for (int w8 = 1; w8 < 8; ++w8) {
+            const float x = s.red6[w8][tid];
             acc = tid == 1 ? fminf(acc, x) : tid == 2 ? fmaxf(acc, x) : acc + x;
           }
           // the item's record slot; the unit's first record also fills every
