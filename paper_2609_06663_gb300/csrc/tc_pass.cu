@@ -52,8 +52,9 @@
 // items; warps 12-15 (key warps, one key per thread) compute the key norms of
 // every tile as it lands (the sum weights in pass 1, a hand-off to the
 // epilogue in pass 2) and read the chunk sums; warps 4-11 are the epilogue
-// (one key per TMEM lane, window rows split in two halves), which also runs
-// the fold items.  setmaxnreg gives the two epilogue warpgroups 176
+// (one key per TMEM lane; in pass 1 the window rows split in two halves, in
+// pass 2 the tiles: half h takes every row of the item's tiles t with
+// t % 2 == h), which also runs the fold items.  setmaxnreg gives the two epilogue warpgroups 176
 // registers a thread and the others 80.
 // Every mbarrier wait and spin is bounded (a limit in nanoseconds of the
 // global timer): on timeout the kernel records ECOKV_ERR_TIMEOUT, raises a
